@@ -1,0 +1,169 @@
+"""Pins of the oracle's decoding algorithms against what Sec. 3.1 fixes.
+
+* the Jacobi fixed point is the greedy AR output (Sec. 3.1, citing Song et al.);
+* every iteration with KV cache fixes at least one token (Sec. 3.1, "Jacobi
+  decoding with KV cache"), so an n-token window converges in k <= n
+  iterations; vanilla Jacobi (Eq. 3 without cache) needs at most n + 1 passes
+  to observe y^(k) = y^(k-1);
+* a guess that already equals the AR continuation is accepted whole in one step;
+* n = 1 Jacobi is AR, step for step;
+* brute force over every initial block of a micro model: each cached step's
+  accepted count equals the count obtained by evaluating Eq. 3 row by row
+  without any cache.
+"""
+from dataclasses import replace
+
+import numpy as np
+import pytest
+
+from oracle import oracle as orc
+from paper_2403_00835_gb300 import synthetic as syn
+
+MICRO = replace(syn.TINY, name="micro", n_layers=1, d_model=16, n_heads=2, n_kv_heads=2,
+                head_dim=8, ffn=24, vocab=8)
+
+
+def oracle_model(cfg, w):
+    wd = orc.ORC_F32 if cfg.dtype == "f32" else orc.ORC_BF16
+    return orc.OracleModel(orc.OracleArch(**syn.oracle_arch_kwargs(cfg)), w, wd)
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    cfg = syn.TINY
+    return cfg, oracle_model(cfg, syn.make_weights(cfg, seed=0))
+
+
+@pytest.fixture(scope="module")
+def micro():
+    # large init scale so the micro model's argmax is far from uniform
+    return oracle_model(MICRO, syn.make_weights(MICRO, seed=11, std=0.7))
+
+
+@pytest.mark.parametrize("mode", ["refill", "shrink"])
+@pytest.mark.parametrize("n,seed", [(8, 2), (5, 3), (16, 4)])
+def test_jacobi_fixed_point_equals_ar(tiny, mode, n, seed):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    ar = orc.ar_decode(m, prompt, 40)
+    jr = orc.jacobi_decode(m, prompt, n, 40, seed=seed, mode=mode)
+    assert jr.tokens == ar.tokens
+    assert all(a >= 1 for a in jr.accepted)
+    assert sum(jr.accepted) == 40
+    assert jr.iterations == len(jr.accepted) <= 40
+
+
+def test_jacobi_prompt_guesses_fixed_point(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    ar = orc.ar_decode(m, prompt, 24)
+    jr = orc.jacobi_decode(m, prompt, 8, 24, seed=9, guess_init="prompt", record=True)
+    assert jr.tokens == ar.tokens
+    # every initial guess slot is a prompt token
+    assert set(jr.trajectory[0][1:]) <= set(prompt)
+
+
+def test_shrink_window_converges_within_n(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    n = 8
+    jr = orc.jacobi_decode(m, prompt, n, 48, seed=5, mode="shrink", record=True)
+    # windows are delimited by the block width returning to n
+    widths = [len(b) for b in jr.trajectory]
+    windows, cur = [], 0
+    for i, wdt in enumerate(widths):
+        if wdt == n and i > 0:
+            windows.append(cur)
+            cur = 0
+        cur += 1
+    windows.append(cur)
+    assert all(k <= n for k in windows)
+    assert sum(jr.accepted) == 48
+
+
+def test_ar_guess_converges_in_one_step(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    n = 8
+    ar = orc.ar_decode(m, prompt, n + 1)
+    s = m.session(64)
+    head, _, _ = orc.prefill(s, prompt)
+    assert head == ar.tokens[0]
+    st = orc.jacobi_step(s, ar.tokens[:n], len(prompt))
+    assert st.accepted == n
+    assert st.pred[n - 1] == ar.tokens[n]  # the next head is the (n+1)-th AR token
+
+
+def test_n1_jacobi_is_ar(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    ar = orc.ar_decode(m, prompt, 20)
+    jr = orc.jacobi_decode(m, prompt, 1, 20, seed=0)
+    assert jr.tokens == ar.tokens
+    assert jr.accepted == [1] * 20 and jr.iterations == 20
+
+
+def test_eos_stops_decoding(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    ar = orc.ar_decode(m, prompt, 30)
+    eos = ar.tokens[11]
+    first = ar.tokens.index(eos)
+    jr = orc.jacobi_decode(m, prompt, 8, 30, seed=2, eos_id=eos)
+    assert jr.tokens == ar.tokens[: first + 1]
+    assert orc.ar_decode(m, prompt, 30, eos_id=eos).tokens == ar.tokens[: first + 1]
+
+
+def test_vanilla_jacobi_fixed_point(tiny):
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [12], seed=4)[0]
+    n = 6
+    ar = orc.ar_decode(m, prompt, n)
+    for seed in range(3):
+        y0 = syn.make_guesses(cfg.vocab, 1, n, seed=seed)[0]
+        ystar, k = orc.jacobi_vanilla(m, prompt, y0)
+        assert ystar == ar.tokens
+        assert 1 <= k <= n + 1
+
+
+def _definitional_accept(model, prompt, block):
+    """Longest prefix of the block that Eq. 3's rows reproduce, each row
+    evaluated by a fresh full forward of [x; block_<i] (no cache reuse)."""
+    a = 1
+    while a < len(block):
+        seq = list(prompt) + list(block[:a])
+        row = model.session(len(seq)).forward(seq, 0, rows=[len(seq) - 1])[0]
+        if int(np.argmax(row)) != block[a]:
+            break
+        a += 1
+    return a
+
+
+def test_brute_force_micro_model(micro):
+    m = micro
+    V, n = MICRO.vocab, 3
+    prompt = [3, 1, 4, 1, 5]
+    ar = orc.ar_decode(m, prompt, n + 2)
+    s0 = m.session(16)
+    head, _, _ = orc.prefill(s0, prompt)
+    assert head == ar.tokens[0]
+    seen_a = set()
+    for g1 in range(V):
+        for g2 in range(V):
+            block = [head, g1, g2]
+            s = m.session(16)
+            s.forward(prompt, 0, rows=[])
+            st = orc.jacobi_step(s, block, len(prompt))
+            assert st.accepted == _definitional_accept(m, prompt, block)
+            seen_a.add(st.accepted)
+    assert seen_a == {1, 2, 3}
+    # vanilla Jacobi from every one of the V^n initial blocks reaches the AR output
+    for idx in range(V ** n):
+        y0 = [(idx // V ** i) % V for i in range(n)]
+        ystar, k = orc.jacobi_vanilla(m, prompt, y0)
+        assert ystar == ar.tokens[:n] and k <= n + 1
+    # full decodes from several guess streams, both block policies
+    for seed in range(8):
+        for mode in ("refill", "shrink"):
+            assert orc.jacobi_decode(m, prompt, n, 12, seed=seed, mode=mode).tokens == \
+                orc.ar_decode(m, prompt, 12).tokens
