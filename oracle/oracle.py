@@ -327,6 +327,7 @@ class DecodeResult:
     iterations: int
     accepted: list = field(default_factory=list)   # a per iteration
     min_gap: list = field(default_factory=list)    # per iteration: min gap over the committed rows' predictions
+    min_gap_all: list = field(default_factory=list)  # per iteration: min gap over every row of the block
     trajectory: list = field(default_factory=list)  # blocks fed to each iteration
 
 
@@ -386,6 +387,7 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
         res.tokens += block[:a]
         res.accepted.append(a)
         res.min_gap.append(min(st.gap[:a]))
+        res.min_gap_all.append(min(st.gap))
         L += a
         res.iterations += 1
         if stop or len(res.tokens) >= max_new:

@@ -1,0 +1,171 @@
+// Internal declarations shared by the kernels and the host engine.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace cllm {
+
+// Device error bits (the device status word); never __trap()/assert.
+enum : int {
+  DERR_TOKEN = 1,     // a token id outside [0, vocab)
+  DERR_CAPACITY = 2,  // a position at or past max_seq
+  DERR_TIMEOUT = 4,   // a bounded wait ran out
+  DERR_SHAPE = 8,     // an internal shape check failed
+};
+
+constexpr int kAttnChunk = 128;  // keys per attention chunk, anchored at absolute positions
+constexpr int kQTile = 16;       // query rows per attention tile
+constexpr int kBK = 64;          // K elements per pipeline stage (128 B of bf16)
+constexpr int kBM = 128;         // weight rows per tile (MMA M)
+constexpr int kEpiCols = 16;     // columns per epilogue chunk
+
+enum EpiKind : int { EPI_QKV = 0, EPI_GATEUP = 1, EPI_RESID = 2, EPI_ARGMAX = 3 };
+
+// Per-launch epilogue arguments (passed by value; one struct for all kinds).
+struct EpiArgs {
+  int T;      // valid token rows of this launch
+  int ldt;    // row stride (tokens) of the per-token partial arrays (ssq, argmax)
+  // RMSNorm scale of the GEMM input: rs[t] = 1/sqrt(sum_i ssq_in[i*ldt+t] / d + eps)
+  const float* ssq_in;
+  int ssq_tiles;
+  float inv_d, eps;
+  // QKV: rotate-half RoPE, Q out, K/V into the cache at (bidx[t], pos[t])
+  void* q_out;
+  void* k_cache;  // this layer's [B][Hkv][max_seq][hd]
+  void* v_cache;
+  int dq, dkv, hd, n_kv_heads, max_seq;
+  const int* pos;
+  const int* bidx;
+  const float2* rope;  // [max_seq][hd/2] (cos, sin)
+  // GATEUP: h[t][f] = silu(gate) * up
+  void* h_out;
+  int F;
+  // RESID: x += D; xg = x * gnext; ssq_out per 128-row tile
+  float* x;
+  void* xg;
+  const void* gnext;
+  float* ssq_out;
+  int d;
+  // ARGMAX: per-tile (max, argmax, second max); last unit reduces to pred/gap
+  float* am_part;  // [mtiles][ldt][3]
+  int* am_ticket;
+  int am_units;
+  int am_mtiles;
+  int* pred;
+  float* gap;
+  float* logits;  // optional debug [T][V]
+  int V;
+  int* err;
+};
+
+// Work decomposition of one weight-streaming GEMM launch.
+//   D[m][t] = sum_k W[m][k] X[t][k]  (m: weight rows, t: tokens)
+// The chunk space (unit, k-chunk) is split into contiguous ranges of `cpc`
+// chunks, one per CTA; a unit is one 128-row tile x one N-tile of tokens.
+struct GemmArgs {
+  int M, K, T;
+  int mtiles, ntiles, kchunks, cpc, bn, maxc;
+  int rows_q, rows_qk;  // QKV: first rows of the K and V sections (weight-map select)
+  float* partial;       // [units*maxc][bn][128] split-K partial tiles
+  int* tickets;         // [units] arrival counters (self-resetting)
+  // SIMT (fp32) path only
+  const void* A0;
+  const void* A1;
+  const void* A2;
+  const void* X;
+  int ldx;
+  int* err;
+};
+
+struct AttnArgs {
+  const void* q;        // [T][n_heads*hd]
+  const void* k_cache;  // this layer's [B][Hkv][max_seq][hd]
+  const void* v_cache;
+  const int* seq_start;  // [B] position of the sequence's first row
+  const int* seq_row0;   // [B] index of the sequence's first row
+  const int* seq_nrows;  // [B]
+  const int2* qtiles;    // (b, first row within sequence) per 16-row query tile
+  int n_qtiles;
+  int H, Hkv, hd, max_seq, nch_max;
+  float scale_log2;   // log2(e) / sqrt(hd)
+  float* part_o;      // [row][H][nch_max][hd], unnormalised
+  float2* part_ml;    // [row][H][nch_max]: (running max in log2 units, sum)
+  const int* pos;     // [T]
+  void* out;          // [T][H*hd]
+  int T;
+  int* err;
+};
+
+struct EmbedArgs {
+  const void* emb;    // [V][d]
+  const void* gain;   // first layer's attention-norm gain [d]
+  int V, d, T, ldt;
+  // step mode (block != nullptr): row t = b*n + k, token block[b][k], position L[b] + k
+  const int* block;
+  const int* L;
+  int n, B, max_seq;
+  // prefill mode: per-row token / position / sequence given
+  const int* tok_in;
+  const int* pos_in;
+  const int* bidx_in;
+  // outputs
+  float* x;
+  void* xg;
+  float* ssq;  // [d/128][ldt]
+  int* pos;
+  int* bidx;
+  int* seq_start;
+  int* seq_row0;
+  int* seq_nrows;
+  int* err;
+};
+
+struct AcceptArgs {
+  int B, n, V;
+  int decode;  // 1: decode loop (commit to out, done flags, refill); 0: single step
+  int max_new, eos;
+  unsigned long long seed;
+  int guess_mode;
+  const int* pred;  // [B*n]
+  int* block;       // [B][n]
+  int* L;
+  int* head;
+  int* committed;
+  int* iters;
+  int* done;
+  int* out;  // [B][max_new]
+  int* accepted;
+  const int* prompts;  // [B][max_seq]
+  const int* plen;
+  int prompt_ld;
+  int* status;  // [0] active sequences, [1] tokens committed by this iteration
+};
+
+// ---- launchers (kernels.cu) --------------------------------------------------------
+struct GemmMaps {
+  CUtensorMap a0, a1, a2, b;
+};
+
+cudaError_t launch_embed(const EmbedArgs& a, int act_bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_gemm_tc(int kind, int bn_max, const GemmMaps& maps, const GemmArgs& g,
+                           const EpiArgs& e, int grid, cudaStream_t s, bool pdl);
+cudaError_t launch_gemm_simt(int kind, const GemmArgs& g, const EpiArgs& e, cudaStream_t s,
+                             bool pdl);
+cudaError_t launch_attention(const AttnArgs& a, int act_bf16, int grid, cudaStream_t s, bool pdl);
+cudaError_t launch_attn_combine(const AttnArgs& a, int act_bf16, cudaStream_t s, bool pdl);
+cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s, bool pdl);
+cudaError_t launch_decode_init(const AcceptArgs& a, cudaStream_t s);
+cudaError_t launch_set_head(int* block, const int* head, int B, int n, int V, int* err,
+                            cudaStream_t s);
+cudaError_t launch_gather_rows(const void* xg_src, const float* ssq_src, void* xg_dst,
+                               float* ssq_dst, const int* rows, int B, int d, int ldt_src,
+                               int ldt_dst, int act_bf16, cudaStream_t s);
+int gemm_tc_stages(int bn_max);
+size_t gemm_tc_smem_bytes(int bn_max);
+cudaError_t gemm_tc_set_attributes();
+cudaError_t attention_set_attributes();
+size_t attention_smem_bytes(int act_bf16, int hd);
+
+}  // namespace cllm
