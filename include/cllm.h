@@ -43,8 +43,10 @@ extern "C" {
 #define CLLM_EUNSUPPORTED -8 /* shape or device this build does not handle          */
 
 /* ---- element types ----------------------------------------------------------- */
-#define CLLM_F32 0   /* fp32 weights and activations (parity configurations)        */
-#define CLLM_BF16 1  /* bf16 weights, bf16 GEMM inputs, fp32 accumulation/residual  */
+#define CLLM_F32 0   /* fp32 weights and activations (parity configurations)         */
+#define CLLM_BF16 1  /* bf16 weights; every GEMM input carried as two bf16 planes     */
+                     /* (hi + lo), fp32 accumulation and residual stream; Q, K, V and */
+                     /* the attention probabilities in fp16 with fp32 accumulation    */
 
 /* ---- decode options ---------------------------------------------------------- */
 #define CLLM_GUESS_UNIFORM 0      /* initial/refill guesses uniform over the vocab   */
@@ -96,7 +98,8 @@ typedef struct cllm_ctx cllm_ctx;
 
 /*
  * Create a context: validates the shape, builds the TMA descriptors of the
- * weights, and allocates (owns) the KV cache K,V[layer][b][kv_head][pos][hd],
+ * weights, and allocates (owns) the KV cache K,V[layer][b][kv_head][pos][hd]
+ * (fp32 for CLLM_F32, fp16 for CLLM_BF16),
  * the activation scratch and the device status word.  cuda_stream is a
  * cudaStream_t (NULL = a stream the context creates and owns).  The current
  * device at the call is the context's device.

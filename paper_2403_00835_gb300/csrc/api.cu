@@ -112,6 +112,7 @@ struct cllm_ctx {
   size_t esz = 2;
   int d = 0, H = 0, Hkv = 0, hd = 0, dq = 0, dkv = 0, F = 0, V = 0, NL = 0;
   int Tcap = 0, prefill_cap = 0, nch_max = 0, max_qtiles = 0;
+  int planes = 1;  // GEMM activation planes: 2 (bf16 hi + lo) in the bf16 engine
   // weights
   const void *tok_emb = nullptr, *final_norm = nullptr, *lm_head = nullptr;
   CUtensorMap mlm{};
@@ -222,6 +223,8 @@ EpiArgs base_epi(cllm_ctx* c, int T) {
   e.d = c->d;
   e.V = c->V;
   e.err = c->err;
+  e.plane_x = c->planes == 2 ? static_cast<size_t>(c->Tcap) * c->d : 0;
+  e.plane_h = c->planes == 2 ? static_cast<size_t>(c->Tcap) * c->F : 0;
   return e;
 }
 
@@ -239,6 +242,7 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
   g.err = c->err;
   g.tickets = c->tickets;
   g.partial = c->gemm_part;
+  g.lo_rows = c->Tcap;
   cudaError_t err;
   if (!c->bf16) {
     g.mtiles = mtiles;
@@ -266,7 +270,7 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
     maps.a0 = *m0;
     maps.a1 = m1 ? *m1 : *m0;
     maps.a2 = m2 ? *m2 : *m0;
-    if (!make_map(&maps.b, X, static_cast<uint64_t>(K), static_cast<uint64_t>(c->Tcap),
+    if (!make_map(&maps.b, X, static_cast<uint64_t>(K), static_cast<uint64_t>(2 * c->Tcap),
                   static_cast<uint32_t>(p.bn)))
       return cudaErrorInvalidValue;
     EpiArgs ee = e;
@@ -315,6 +319,7 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
   }
   ea.x = c->x;
   ea.xg = c->xg;
+  ea.plane = c->planes == 2 ? static_cast<size_t>(c->Tcap) * c->d : 0;
   ea.ssq = c->ssq;
   ea.pos = c->pos;
   ea.bidx = c->bidx;
@@ -341,6 +346,7 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
   aa.part_ml = c->part_ml;
   aa.pos = c->pos;
   aa.out = c->attn;
+  aa.plane_out = c->planes == 2 ? static_cast<size_t>(c->Tcap) * c->dq : 0;
   aa.T = T;
   aa.err = c->err;
 
@@ -405,7 +411,10 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
   if (f.mode == MODE_PREFILL) {
     if ((err = after_launch(c, s, "gather",
                             launch_gather_rows(c->xg, c->ssq, c->xg_last, c->ssq_last, c->last_rows,
-                                               f.n_last, c->d, c->Tcap, c->Tcap, ab, s))) !=
+                                               f.n_last, c->d, c->Tcap, c->Tcap,
+                                               static_cast<size_t>(c->Tcap) * c->d * (c->planes - 1),
+                                               static_cast<size_t>(c->Tcap) * c->d * (c->planes - 1),
+                                               ab, s))) !=
         cudaSuccess)
       return err;
     e.T = f.n_last;
@@ -640,6 +649,7 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
   c->sms = prop.multiProcessorCount;
   c->bf16 = a.dtype == CLLM_BF16;
   c->esz = c->bf16 ? 2 : 4;
+  c->planes = c->bf16 ? 2 : 1;
   c->d = a.d_model;
   c->H = a.n_heads;
   c->Hkv = a.n_kv_heads;
@@ -716,12 +726,13 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
     c->max_qtiles = c->Tcap / kQTile + a.max_batch;
     const size_t T = c->Tcap;
     const size_t es = c->esz;
+    const size_t P = c->planes;
     const int dmax = std::max(c->dq, std::max(c->d, c->F));
     (void)dmax;
-    bool ok = dev_alloc(c, &c->x, T * c->d * 4) && dev_alloc(c, &c->xg, T * c->d * es) &&
+    bool ok = dev_alloc(c, &c->x, T * c->d * 4) && dev_alloc(c, &c->xg, P * T * c->d * es) &&
               dev_alloc(c, &c->ssq, (c->d / kBM) * T * 4) && dev_alloc(c, &c->q, T * c->dq * es) &&
-              dev_alloc(c, &c->attn, T * c->dq * es) && dev_alloc(c, &c->h, T * c->F * es) &&
-              dev_alloc(c, &c->xg_last, T * c->d * es) &&
+              dev_alloc(c, &c->attn, P * T * c->dq * es) && dev_alloc(c, &c->h, P * T * c->F * es) &&
+              dev_alloc(c, &c->xg_last, P * T * c->d * es) &&
               dev_alloc(c, &c->ssq_last, (c->d / kBM) * T * 4) &&
               dev_alloc(c, &c->last_rows, a.max_batch * 4);
     if (!ok) {
@@ -1160,7 +1171,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
   const Part p = plan_gemm(mtiles, K, T, prop.multiProcessorCount);
   const int ldt = round_up(T, 16);
   GemmMaps maps{};
-  if (!make_map(&maps.a0, W, K, M, kBM) || !make_map(&maps.b, X, K, x_rows, p.bn))
+  if (!make_map(&maps.a0, W, K, M, kBM) || !make_map(&maps.b, X, K, 2 * x_rows, p.bn))
     return CLLM_EINVAL;
   maps.a1 = maps.a2 = maps.a0;
   std::vector<void*> tmp;
@@ -1176,7 +1187,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     int* tickets = static_cast<int*>(alloc(mtiles * 4));
     int* err = static_cast<int*>(alloc(16));
     float* ssq = static_cast<float*>(alloc(static_cast<size_t>(mtiles) * ldt * 4));
-    void* xg = alloc(static_cast<size_t>(T) * M * 2);
+    void* xg = alloc(static_cast<size_t>(T) * M * 2 * 2);
     __nv_bfloat16* ones = static_cast<__nv_bfloat16*>(alloc(static_cast<size_t>(M) * 2));
     if (!part || !tickets || !err || !ssq || !xg || !ones) {
       rc = CLLM_ENOMEM;
@@ -1199,6 +1210,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     g.maxc = p.maxc;
     g.rows_q = M;
     g.rows_qk = M;
+    g.lo_rows = x_rows;
     g.partial = part;
     g.tickets = tickets;
     g.err = err;
@@ -1208,6 +1220,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     e.x = Y;
     e.xg = xg;
     e.gnext = ones;
+    e.plane_x = static_cast<size_t>(T) * M;
     e.ssq_out = ssq;
     e.d = M;
     e.err = err;

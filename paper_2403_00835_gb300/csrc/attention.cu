@@ -11,8 +11,9 @@
 // only on its own position, query and keys, not on how many rows share the
 // step, so a Jacobi step and an AR step produce the same bits for a token.
 //
-// bf16: each of 4 warps takes 32 keys of the chunk for the tile's 16 rows;
-// S = Q K^T and O = P V run on mma.sync m16n8k16 (fp32 accumulate) with
+// bf16 engine (Q, K, V and P held in fp16): each of 4 warps takes 32 keys of
+// the chunk for the tile's 16 rows; S = Q K^T and O = P V run on mma.sync
+// m16n8k16 f16 x f16 -> fp32 with
 // ldmatrix loads from padded shared memory; the softmax is computed on the
 // accumulator fragments with quad shuffles; the 4 warps' partials are merged
 // in warp order.  fp32: a SIMT kernel with a per-row online softmax.
@@ -69,10 +70,10 @@ __device__ __forceinline__ int attn_find_qtile(const int* pre, int n, int item) 
 }
 
 template <int HD>
-struct AttnSmemBf16 {
-  __nv_bfloat16 q[kQTile][HD + 8];
-  __nv_bfloat16 k[kAttnChunk][HD + 8];  // reused as float co[4][kQTile][HD] for the warp merge
-  __nv_bfloat16 v[kAttnChunk][HD + 8];
+struct AttnSmemF16 {
+  __half q[kQTile][HD + 8];
+  __half k[kAttnChunk][HD + 8];  // reused as float co[4][kQTile][HD] for the warp merge
+  __half v[kAttnChunk][HD + 8];
   float m[4][kQTile];
   float l[4][kQTile];
   int pre[kMaxQTilesSmem + 1];
@@ -80,10 +81,10 @@ struct AttnSmemBf16 {
 
 template <int HD>
 __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
-  static_assert(sizeof(float) * 4 * kQTile * HD <= sizeof(__nv_bfloat16) * kAttnChunk * (HD + 8),
+  static_assert(sizeof(float) * 4 * kQTile * HD <= sizeof(__half) * kAttnChunk * (HD + 8),
                 "merge area must fit in the K tile");
-  extern __shared__ uint8_t smem_raw[];
-  AttnSmemBf16<HD>& sm = *reinterpret_cast<AttnSmemBf16<HD>*>(smem_raw);
+  extern __shared__ __align__(16) uint8_t smem_raw[];
+  AttnSmemF16<HD>& sm = *reinterpret_cast<AttnSmemF16<HD>*>(smem_raw);
   pdl_launch_dependents();
   pdl_wait();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -91,9 +92,9 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
   const int total = attn_item_prefix(a, sm.pre);
   const int group = a.H / a.Hkv;
   const int ldq = a.H * HD;
-  const __nv_bfloat16* Q = static_cast<const __nv_bfloat16*>(a.q);
-  const __nv_bfloat16* KC = static_cast<const __nv_bfloat16*>(a.k_cache);
-  const __nv_bfloat16* VC = static_cast<const __nv_bfloat16*>(a.v_cache);
+  const __half* Q = static_cast<const __half*>(a.q);
+  const __half* KC = static_cast<const __half*>(a.k_cache);
+  const __half* VC = static_cast<const __half*>(a.v_cache);
   float (*co)[kQTile][HD] = reinterpret_cast<float (*)[kQTile][HD]>(&sm.k[0][0]);
 
   for (int item = blockIdx.x; item < total; item += gridDim.x) {
@@ -163,8 +164,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
           uint32_t kb4[4];
           const int mi = lane >> 3;
           ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
-          mma_bf16_16816(s[j], qa0, kb4[0], kb4[1]);
-          mma_bf16_16816(s[j], qa1, kb4[2], kb4[3]);
+          mma_f16_16816(s[j], qa0, kb4[0], kb4[1]);
+          mma_f16_16816(s[j], qa1, kb4[2], kb4[3]);
         }
       }
       // mask + scale (log2 domain)
@@ -195,8 +196,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
         const float p2 = exp2f(s[j][2] - uB), p3 = exp2f(s[j][3] - uB);
         lA += p0 + p1;
         lB += p2 + p3;
-        pa[j >> 1][(j & 1) * 2 + 0] = pack_bf16x2(p0, p1);
-        pa[j >> 1][(j & 1) * 2 + 1] = pack_bf16x2(p2, p3);
+        pa[j >> 1][(j & 1) * 2 + 0] = pack_f16x2(p0, p1);
+        pa[j >> 1][(j & 1) * 2 + 1] = pack_f16x2(p2, p3);
       }
       lA += __shfl_xor_sync(0xffffffffu, lA, 1);
       lA += __shfl_xor_sync(0xffffffffu, lA, 2);
@@ -212,8 +213,8 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
           uint32_t vb[4];
           const int mi = lane >> 3;
           ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
-          mma_bf16_16816(o[dn], af, vb[0], vb[1]);
-          mma_bf16_16816(o[dn + 1], af, vb[2], vb[3]);
+          mma_f16_16816(o[dn], af, vb[0], vb[1]);
+          mma_f16_16816(o[dn + 1], af, vb[2], vb[3]);
         }
       }
     }
@@ -348,7 +349,8 @@ __global__ void attn_combine_kernel(const AttnArgs a) {
       l += f * ml.y;
       acc += f * a.part_o[(base + c) * a.hd + d];
     }
-    st_act(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * a.hd + h * a.hd + d, acc / l);
+    st_gin(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * a.hd + h * a.hd + d, a.plane_out,
+           acc / l);
   }
 }
 
@@ -356,16 +358,22 @@ __global__ void attn_combine_kernel(const AttnArgs a) {
 
 size_t attention_smem_bytes(int act_bf16, int hd) {
   if (!act_bf16) return 0;
-  return hd == 64 ? sizeof(AttnSmemBf16<64>) : sizeof(AttnSmemBf16<128>);
+  return hd == 64 ? sizeof(AttnSmemF16<64>) : sizeof(AttnSmemF16<128>);
 }
 
 cudaError_t attention_set_attributes() {
   cudaError_t e = cudaFuncSetAttribute(attn_chunk_mma_kernel<64>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(sizeof(AttnSmemBf16<64>)));
+                                       static_cast<int>(sizeof(AttnSmemF16<64>)));
   if (e != cudaSuccess) return e;
+  for (const void* k : {reinterpret_cast<const void*>(attn_chunk_mma_kernel<64>),
+                        reinterpret_cast<const void*>(attn_chunk_mma_kernel<128>)}) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             static_cast<int>(cudaSharedmemCarveoutMaxShared));
+    if (e != cudaSuccess) return e;
+  }
   return cudaFuncSetAttribute(attn_chunk_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(sizeof(AttnSmemBf16<128>)));
+                              static_cast<int>(sizeof(AttnSmemF16<128>)));
 }
 
 static void attn_cfg(cudaLaunchConfig_t& cfg, cudaLaunchAttribute* attr, dim3 grid, dim3 block,

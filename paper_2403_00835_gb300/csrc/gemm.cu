@@ -107,8 +107,9 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
     for (int j = 0; j < kEpiCols; ++j) {
       const int t = t0 + j;
       if (t >= e.T) continue;
+      using AT = typename AttnType<Act>::T;
       if (sec == 0) {
-        st_act(reinterpret_cast<Act*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
+        st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
       } else {
         const int p = e.pos[t], b = e.bidx[t];
         if (p < 0 || p >= e.max_seq) {
@@ -117,7 +118,7 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
         }
         const size_t off =
             ((static_cast<size_t>(b) * e.n_kv_heads + head) * e.max_seq + p) * e.hd + i;
-        st_act(reinterpret_cast<Act*>(sec == 1 ? e.k_cache : e.v_cache), off, v[j]);
+        st_act(reinterpret_cast<AT*>(sec == 1 ? e.k_cache : e.v_cache), off, v[j]);
       }
     }
   } else if (KIND == EPI_GATEUP) {
@@ -136,7 +137,7 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
           const int t = t0 + j;
           if (t < e.T) {
             const float gt = v[j], up = s.x[j][r + 64];
-            st_act(reinterpret_cast<Act*>(e.h_out), static_cast<size_t>(t) * e.F + f,
+            st_gin(reinterpret_cast<Act*>(e.h_out), static_cast<size_t>(t) * e.F + f, e.plane_h,
                    gt / (1.f + expf(-gt)) * up);
           }
         }
@@ -154,7 +155,7 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
         const size_t o = static_cast<size_t>(t) * e.d + m;
         const float xi = e.x[o] + v[j];
         e.x[o] = xi;
-        st_act(reinterpret_cast<Act*>(e.xg), o, xi * gn);
+        st_gin(reinterpret_cast<Act*>(e.xg), o, e.plane_x, xi * gn);
         sq = xi * xi;
       }
       sq = warp_sum(sq);
@@ -254,11 +255,15 @@ __device__ void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
 // tcgen05 kernel (bf16)
 // ---------------------------------------------------------------------------------
 
+// Stage = one 128 x 64 weight tile + the hi and lo planes of a BNMAX x 64
+// activation tile.  Up to BNMAX = 64 two CTAs fit on an SM (so the next
+// kernel's CTAs can start while this one drains).
 template <int BNMAX>
 struct TcCfg {
-  static constexpr int STAGES = BNMAX <= 32 ? 5 : (BNMAX <= 64 ? 4 : (BNMAX <= 128 ? 3 : 4));
+  static constexpr int STAGES = BNMAX <= 32 ? 4 : (BNMAX <= 64 ? 3 : (BNMAX <= 128 ? 3 : 2));
   static constexpr int A_BYTES = kBM * kBK * 2;
-  static constexpr int B_BYTES = BNMAX * kBK * 2;
+  static constexpr int B_HALF = BNMAX * kBK * 2;
+  static constexpr int B_BYTES = 2 * B_HALF;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
   static constexpr int TMEM_COLS = 2 * BNMAX;  // two accumulators: 64, 128, 256 or 512
   static constexpr size_t BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
@@ -269,6 +274,10 @@ struct TcCfg {
 struct Segment {
   int unit, k0, k1;
 };
+
+// Weight tiles per CTA prefetched into L2 ahead of the shared-memory ring
+// (16 x 16 KB x 152 CTAs ~ 40 MB of the 129 MB L2).
+constexpr int kL2Ahead = 16;
 
 // Iterate the (unit, k-range) segments of the chunk range [c, c1).
 __device__ __forceinline__ bool next_segment(int& c, int c1, int kchunks, Segment& sg) {
@@ -340,7 +349,7 @@ __global__ void __launch_bounds__(192, 1)
   const int c0 = blockIdx.x * g.cpc;
   const int c1 = min(total, c0 + g.cpc);
   const bool tile_mode = g.ntiles > 1;
-  const uint32_t b_bytes = static_cast<uint32_t>(g.bn) * kBK * 2;
+  const uint32_t b_bytes = 2u * static_cast<uint32_t>(g.bn) * kBK * 2;
 
   if (warp == 0) {
     if (lane == 0 && c0 < c1) {
@@ -375,15 +384,37 @@ __global__ void __launch_bounds__(192, 1)
         const int u = unit_of(c), k = c - u * g.kchunks;
         const int nt = u % g.ntiles;
         const int st = idx % S;
-        tma_load_2d(sB + st * Cfg::B_BYTES, &mB, &full[st], k * kBK, tile_mode ? nt * BNMAX : 0,
-                    pol_x);
+        const int row0 = tile_mode ? nt * BNMAX : 0;
+        uint8_t* dst = sB + st * Cfg::B_BYTES;
+        tma_load_2d(dst, &mB, &full[st], k * kBK, row0, pol_x);
+        tma_load_2d(dst + Cfg::B_HALF, &mB, &full[st], k * kBK, g.lo_rows + row0, pol_x);
       };
       // Weights do not depend on earlier kernels: start streaming them before
-      // waiting for the previous kernel (programmatic dependent launch).
+      // waiting for the previous kernel (programmatic dependent launch) --
+      // the first S tiles into shared memory, the next kL2Ahead into L2.
       const int pre = min(S, nchunks);
       for (int idx = 0; idx < pre; ++idx) {
         mbar_arrive_expect_tx(&full[idx], Cfg::A_BYTES + b_bytes);
         load_a(idx);
+      }
+      for (int idx = pre; idx < min(nchunks, pre + kL2Ahead); ++idx) {
+        const int c = c0 + idx;
+        const int u = unit_of(c), k = c - u * g.kchunks;
+        const int mt = u / g.ntiles;
+        if (KIND == EPI_GATEUP) {
+          tma_prefetch_l2_2d(&mA0, k * kBK, mt * 64);
+          tma_prefetch_l2_2d(&mA1, k * kBK, mt * 64);
+        } else if (KIND == EPI_QKV) {
+          const int row = mt * kBM;
+          if (row < g.rows_q)
+            tma_prefetch_l2_2d(&mA0, k * kBK, row);
+          else if (row < g.rows_qk)
+            tma_prefetch_l2_2d(&mA1, k * kBK, row - g.rows_q);
+          else
+            tma_prefetch_l2_2d(&mA2, k * kBK, row - g.rows_qk);
+        } else {
+          tma_prefetch_l2_2d(&mA0, k * kBK, mt * kBM);
+        }
       }
       pdl_wait();
       for (int idx = 0; idx < pre; ++idx) load_b(idx);
@@ -426,8 +457,10 @@ __global__ void __launch_bounds__(192, 1)
           const uint32_t b_addr = smem_u32(sB + st * Cfg::B_BYTES);
 #pragma unroll
           for (int kk = 0; kk < kBK / 16; ++kk) {
-            tc_mma_f16(dt, sdesc_kmajor_sw128(a_addr + kk * 32), sdesc_kmajor_sw128(b_addr + kk * 32),
-                       idesc, (k > sg.k0 || kk > 0) ? 1u : 0u);
+            const uint64_t ad = sdesc_kmajor_sw128(a_addr + kk * 32);
+            tc_mma_f16(dt, ad, sdesc_kmajor_sw128(b_addr + kk * 32), idesc,
+                       (k > sg.k0 || kk > 0) ? 1u : 0u);
+            tc_mma_f16(dt, ad, sdesc_kmajor_sw128(b_addr + Cfg::B_HALF + kk * 32), idesc, 1u);
           }
           tc_commit(&empty[st]);
         }
@@ -612,8 +645,13 @@ size_t gemm_tc_smem_bytes(int bn_max) {
 
 template <int KIND, int BN>
 static cudaError_t set_attr_one() {
-  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(TcCfg<BN>::SMEM));
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<KIND, BN>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(TcCfg<BN>::SMEM));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemm_tc_kernel<KIND, BN>,
+                              cudaFuncAttributePreferredSharedMemoryCarveout,
+                              static_cast<int>(cudaSharedmemCarveoutMaxShared));
 }
 
 template <int KIND>

@@ -42,12 +42,14 @@ struct EpiArgs {
   // GATEUP: h[t][f] = silu(gate) * up
   void* h_out;
   int F;
+  size_t plane_h;  // element offset of h's lo plane (bf16 engine)
   // RESID: x += D; xg = x * gnext; ssq_out per 128-row tile
   float* x;
   void* xg;
   const void* gnext;
   float* ssq_out;
   int d;
+  size_t plane_x;  // element offset of xg's lo plane (bf16 engine)
   // ARGMAX: per-tile (max, argmax, second max); last unit reduces to pred/gap
   float* am_part;  // [mtiles][ldt][3]
   int* am_ticket;
@@ -68,6 +70,7 @@ struct GemmArgs {
   int M, K, T;
   int mtiles, ntiles, kchunks, cpc, bn, maxc;
   int rows_q, rows_qk;  // QKV: first rows of the K and V sections (weight-map select)
+  int lo_rows;          // row offset of the activations' lo plane in the B map
   float* partial;       // [units*maxc][bn][128] split-K partial tiles
   int* tickets;         // [units] arrival counters (self-resetting)
   // SIMT (fp32) path only
@@ -93,7 +96,8 @@ struct AttnArgs {
   float* part_o;      // [row][H][nch_max][hd], unnormalised
   float2* part_ml;    // [row][H][nch_max]: (running max in log2 units, sum)
   const int* pos;     // [T]
-  void* out;          // [T][H*hd]
+  void* out;          // [T][H*hd] (+ lo plane in the bf16 engine)
+  size_t plane_out;
   int T;
   int* err;
 };
@@ -113,6 +117,7 @@ struct EmbedArgs {
   // outputs
   float* x;
   void* xg;
+  size_t plane;  // element offset of xg's lo plane (bf16 engine)
   float* ssq;  // [d/128][ldt]
   int* pos;
   int* bidx;
@@ -161,7 +166,8 @@ cudaError_t launch_set_head(int* block, const int* head, int B, int n, int V, in
                             cudaStream_t s);
 cudaError_t launch_gather_rows(const void* xg_src, const float* ssq_src, void* xg_dst,
                                float* ssq_dst, const int* rows, int B, int d, int ldt_src,
-                               int ldt_dst, int act_bf16, cudaStream_t s);
+                               int ldt_dst, size_t plane_src, size_t plane_dst, int act_bf16,
+                               cudaStream_t s);
 int gemm_tc_stages(int bn_max);
 size_t gemm_tc_smem_bytes(int bn_max);
 cudaError_t gemm_tc_set_attributes();

@@ -56,7 +56,7 @@ __global__ void __launch_bounds__(128) embed_kernel(const EmbedArgs a) {
   const float e = ld_act(static_cast<const Act*>(a.emb), static_cast<size_t>(tok) * a.d + m);
   const size_t o = static_cast<size_t>(t) * a.d + m;
   a.x[o] = e;
-  st_act(static_cast<Act*>(a.xg), o, e * ld_act(static_cast<const Act*>(a.gain), m));
+  st_gin(static_cast<Act*>(a.xg), o, a.plane, e * ld_act(static_cast<const Act*>(a.gain), m));
   __shared__ float red[4];
   const float s = warp_sum(e * e);
   if ((i & 31) == 0) red[i >> 5] = s;
@@ -167,11 +167,15 @@ __global__ void set_head_kernel(int* block, const int* head, int B, int n, int V
 template <typename Act>
 __global__ void gather_rows_kernel(const Act* xg_src, const float* ssq_src, Act* xg_dst,
                                    float* ssq_dst, const int* rows, int d, int ldt_src,
-                                   int ldt_dst) {
+                                   int ldt_dst, size_t plane_src, size_t plane_dst) {
   const int b = blockIdx.x;
   const int row = rows[b];
-  for (int m = threadIdx.x; m < d; m += blockDim.x)
+  for (int m = threadIdx.x; m < d; m += blockDim.x) {
     xg_dst[static_cast<size_t>(b) * d + m] = xg_src[static_cast<size_t>(row) * d + m];
+    if (plane_dst)
+      xg_dst[plane_dst + static_cast<size_t>(b) * d + m] =
+          xg_src[plane_src + static_cast<size_t>(row) * d + m];
+  }
   for (int i = threadIdx.x; i < d / 128; i += blockDim.x)
     ssq_dst[static_cast<size_t>(i) * ldt_dst + b] = ssq_src[static_cast<size_t>(i) * ldt_src + row];
 }
@@ -218,15 +222,16 @@ cudaError_t launch_set_head(int* block, const int* head, int B, int n, int V, in
 
 cudaError_t launch_gather_rows(const void* xg_src, const float* ssq_src, void* xg_dst,
                                float* ssq_dst, const int* rows, int B, int d, int ldt_src,
-                               int ldt_dst, int act_bf16, cudaStream_t s) {
+                               int ldt_dst, size_t plane_src, size_t plane_dst, int act_bf16,
+                               cudaStream_t s) {
   if (act_bf16)
     gather_rows_kernel<__nv_bfloat16><<<B, 256, 0, s>>>(
         static_cast<const __nv_bfloat16*>(xg_src), ssq_src, static_cast<__nv_bfloat16*>(xg_dst),
-        ssq_dst, rows, d, ldt_src, ldt_dst);
+        ssq_dst, rows, d, ldt_src, ldt_dst, plane_src, plane_dst);
   else
     gather_rows_kernel<float><<<B, 256, 0, s>>>(static_cast<const float*>(xg_src), ssq_src,
                                                 static_cast<float*>(xg_dst), ssq_dst, rows, d,
-                                                ldt_src, ldt_dst);
+                                                ldt_src, ldt_dst, 0, 0);
   return cudaGetLastError();
 }
 

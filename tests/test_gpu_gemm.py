@@ -23,10 +23,17 @@ def _lib():
     return lib
 
 
-def run_gemm(W, X, T):
+def split_hilo(x):
+    """fp32 activations -> stacked bf16 planes [2][rows][K]: hi = bf16(x), lo = bf16(x - hi)."""
+    hi = x.bfloat16()
+    lo = (x - hi.float()).bfloat16()
+    return torch.stack([hi, lo]).contiguous()
+
+
+def run_gemm(W, X2, T):
     M, K = W.shape
     Y = torch.zeros(T, M, device="cuda", dtype=torch.float32)
-    rc = _lib().cllm_test_gemm_bf16(W.data_ptr(), X.data_ptr(), Y.data_ptr(), M, K, T, X.shape[0])
+    rc = _lib().cllm_test_gemm_bf16(W.data_ptr(), X2.data_ptr(), Y.data_ptr(), M, K, T, X2.shape[1])
     assert rc == 0, cllm.STATUS.get(rc, rc)
     return Y
 
@@ -42,10 +49,10 @@ def x_rows(T):
 def test_gemm_matches_fp64(M, K, T):
     g = torch.Generator(device="cuda").manual_seed(M * 7 + K * 3 + T)
     W = (torch.randn(M, K, device="cuda", generator=g) * 0.02).bfloat16()
-    X = torch.randn(x_rows(T), K, device="cuda", generator=g).bfloat16()
-    Y = run_gemm(W, X, T).cpu().double().numpy()
+    X2 = split_hilo(torch.randn(x_rows(T), K, device="cuda", generator=g))
+    Y = run_gemm(W, X2, T).cpu().double().numpy()
     Wd = W.cpu().double().numpy()
-    Xd = X[:T].cpu().double().numpy()
+    Xd = (X2[0, :T].double() + X2[1, :T].double()).cpu().numpy()
     ref = Xd @ Wd.T
     bound = 1e-5 * (np.abs(Xd) @ np.abs(Wd).T) + 1e-7
     assert (np.abs(Y - ref) <= bound).all(), float((np.abs(Y - ref) / bound).max())
@@ -55,8 +62,8 @@ def test_gemm_matches_fp64(M, K, T):
 def test_gemm_column_independent_of_token_count(M, K):
     g = torch.Generator(device="cuda").manual_seed(5)
     W = (torch.randn(M, K, device="cuda", generator=g) * 0.02).bfloat16()
-    X = torch.randn(256, K, device="cuda", generator=g).bfloat16()
-    ys = {T: run_gemm(W, X, T) for T in (1, 16, 48, 64, 256)}
+    X2 = split_hilo(torch.randn(256, K, device="cuda", generator=g))
+    ys = {T: run_gemm(W, X2, T) for T in (1, 16, 48, 64, 256)}
     for T in (16, 48, 64, 256):
         assert torch.equal(ys[T][:1], ys[1])
     assert torch.equal(ys[64][:48], ys[48])
