@@ -212,6 +212,31 @@ int cllm_kernels_per_iteration(cllm_ctx *ctx, int n);
 /* Committed length L_b of each sequence (host array [B]). */
 int cllm_committed_lengths(cllm_ctx *ctx, int32_t *lens_out);
 
+/* ---- allocation-free GEMM -----------------------------------------------------
+ * The paper has no counterpart of this call; it serves callers that cannot
+ * call cudaMalloc -- code under a caching allocator that has reserved the
+ * device's memory, or a latency-critical path that cannot take the implicit
+ * device synchronisation of cudaMalloc/cudaFree.
+ * Computes, with the library's bf16 weight-streaming GEMM kernel,
+ *   Y[t][m] += sum_k W[m][k] * (Xhi[t][k] + Xlo[t][k])   for t < T, m < M.
+ * W: device bf16 [M][K]; X: device bf16 [2][x_rows][K] (hi plane, then lo
+ * plane), x_rows >= T rounded up to 16 (and >= 256 when T > 256); Y: device
+ * fp32 [T][M], accumulated into.  M a multiple of 128, K a multiple of 8.
+ * cuda_stream: the cudaStream_t to run on (NULL = the legacy default stream);
+ * the call synchronises it before returning.
+ * No memory is allocated: all scratch (split-K partial tiles, arrival tickets,
+ * the device error word, epilogue side outputs) lives in one static device
+ * array of 8 MiB that each device loading the library holds until exit.  Sizes
+ * whose scratch would exceed it return CLLM_ECAPACITY before any launch.  The
+ * first call on a device looks up that array's device address; make it before
+ * any stream capture.  Every call reuses the same array (tickets and the error
+ * word are cleared at the start of each call), so calls that overlap on the
+ * GPU -- from several threads or streams -- race and must not be issued.
+ * Returns CLLM_OK, EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA, EDEVICE or ETIMEOUT.
+ */
+int cllm_gemm_bf16_noalloc(const void *W, const void *X, float *Y, int M, int K, int T,
+                           int x_rows, void *cuda_stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -26,7 +26,7 @@ CLLM_BLOCK_REFILL = 0
 EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode",
            "cllm_ar_decode", "cllm_status_string", "cllm_decode_begin", "cllm_decode_run",
            "cllm_decode_read", "cllm_set_profiling", "cllm_profile_read",
-           "cllm_kernels_per_iteration", "cllm_committed_lengths")
+           "cllm_kernels_per_iteration", "cllm_committed_lengths", "cllm_gemm_bf16_noalloc")
 
 
 class CllmError(RuntimeError):
@@ -99,6 +99,9 @@ def load(build_if_missing: bool = True):
                                       ctypes.POINTER(ctypes.c_int), ctypes.c_int]
     lib.cllm_kernels_per_iteration.argtypes = [vp, ctypes.c_int]
     lib.cllm_committed_lengths.argtypes = [vp, i32p]
+    lib.cllm_gemm_bf16_noalloc.argtypes = [vp, vp, vp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                           ctypes.c_int, vp]
+    lib.cllm_gemm_bf16_noalloc.restype = ctypes.c_int
     for name in ("cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode", "cllm_ar_decode",
                  "cllm_decode_begin", "cllm_decode_run", "cllm_decode_read", "cllm_set_profiling",
                  "cllm_profile_read", "cllm_kernels_per_iteration", "cllm_committed_lengths"):

@@ -20,7 +20,7 @@
 
 using namespace cllm;
 
-namespace {
+namespace cllm {
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
@@ -54,13 +54,6 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int ceil_div(int a, int b) { return (a + b - 1) / b; }
-int round_up(int a, int b) { return ceil_div(a, b) * b; }
-
-struct Part {
-  int mtiles, ntiles, kchunks, cpc, bn, bn_max, maxc, grid;
-};
-
 // Split of one GEMM launch over the SMs.  T <= 256: one N-tile holding every
 // token and the (tile, k-chunk) space cut into equal contiguous ranges; the
 // cut depends on the weight shape and the SM count only.  T > 256: whole
@@ -92,6 +85,10 @@ Part plan_gemm(int mtiles, int K, int T, int sms) {
   }
   return p;
 }
+
+}  // namespace cllm
+
+namespace {
 
 struct LayerW {
   const void *attn_norm, *wq, *wk, *wv, *wo, *mlp_norm, *w_gate, *w_up, *w_down;

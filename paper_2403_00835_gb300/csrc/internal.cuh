@@ -153,6 +153,17 @@ struct GemmMaps {
   CUtensorMap a0, a1, a2, b;
 };
 
+inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
+inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
+
+// Work split of one GEMM launch (api.cu).
+struct Part {
+  int mtiles, ntiles, kchunks, cpc, bn, bn_max, maxc, grid;
+};
+Part plan_gemm(int mtiles, int K, int T, int sms);
+// bf16 [outer][inner] tensor map: 64-column x box_outer-row tiles, 128-byte swizzle.
+bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint32_t box_outer);
+
 cudaError_t launch_embed(const EmbedArgs& a, int act_bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_gemm_tc(int kind, int bn_max, const GemmMaps& maps, const GemmArgs& g,
                            const EpiArgs& e, int grid, cudaStream_t s, bool pdl);
