@@ -27,6 +27,19 @@ extern "C" {
  */
 int cllm_test_gemm_bf16(const void *W, const void *X, float *Y, int M, int K, int T, int x_rows);
 
+/*
+ * Timing of the same kernel in a chain: `iters` launches captured in one CUDA
+ * graph, launch i reading weights W + (i % n_w) * w_stride_bytes (distinct
+ * matrices keep the chain from being served by L2), all accumulating into Y.
+ * pdl: launch with programmatic dependent launch; l2_ahead: weight tiles per
+ * CTA prefetched into L2 before waiting on the previous launch (the engine
+ * uses 16).  T <= 256.  The graph runs once to warm up, then once timed with
+ * CUDA events; *us_per_launch = elapsed / iters.  Returns a CLLM_* status.
+ */
+int cllm_test_gemm_bf16_timed(const void *W, long long w_stride_bytes, int n_w, const void *X,
+                              float *Y, int M, int K, int T, int x_rows, int iters, int pdl,
+                              int l2_ahead, float *us_per_launch);
+
 #ifdef __cplusplus
 }
 #endif

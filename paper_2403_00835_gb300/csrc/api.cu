@@ -20,6 +20,11 @@
 
 using namespace cllm;
 
+// Weight tiles per CTA prefetched into L2 ahead of the shared-memory ring.
+// Measured on chains of GEMM launches: it adds traffic without shortening the
+// chain, so it is off.
+static constexpr int kL2AheadDefault = 0;
+
 namespace cllm {
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -240,6 +245,7 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
   g.tickets = c->tickets;
   g.partial = c->gemm_part;
   g.lo_rows = c->Tcap;
+  g.l2_ahead = kL2AheadDefault;
   cudaError_t err;
   if (!c->bf16) {
     g.mtiles = mtiles;
@@ -1208,6 +1214,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     g.rows_q = M;
     g.rows_qk = M;
     g.lo_rows = x_rows;
+    g.l2_ahead = kL2AheadDefault;
     g.partial = part;
     g.tickets = tickets;
     g.err = err;
@@ -1233,6 +1240,119 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     }
     if (herr) rc = (herr & DERR_TIMEOUT) ? CLLM_ETIMEOUT : CLLM_EDEVICE;
   } while (0);
+  for (void* v : tmp) cudaFree(v);
+  return rc;
+}
+
+extern "C" int cllm_test_gemm_bf16_timed(const void* W, long long w_stride_bytes, int n_w,
+                                         const void* X, float* Y, int M, int K, int T, int x_rows,
+                                         int iters, int pdl, int l2_ahead, float* us_per_launch) {
+  if (!W || !X || !Y || !us_per_launch || M < 128 || M % 128 || K < 8 || K % 8 || T < 1 ||
+      T > 256 || iters < 1 || n_w < 1 || l2_ahead < 0)
+    return CLLM_EINVAL;
+  if (x_rows < round_up(T, 16)) return CLLM_EINVAL;
+  int dev = 0;
+  cudaDeviceProp prop;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess)
+    return CLLM_ECUDA;
+  if (prop.major != 10 || prop.minor != 3) return CLLM_EUNSUPPORTED;
+  if (!get_encode() || gemm_tc_set_attributes() != cudaSuccess) return CLLM_ECUDA;
+  const int mtiles = M / kBM;
+  const Part p = plan_gemm(mtiles, K, T, prop.multiProcessorCount);
+  const int ldt = round_up(T, 16);
+  std::vector<GemmMaps> maps(n_w);
+  for (int i = 0; i < n_w; ++i) {
+    const char* wi = static_cast<const char*>(W) + static_cast<long long>(i) * w_stride_bytes;
+    if (!make_map(&maps[i].a0, wi, K, M, kBM) || !make_map(&maps[i].b, X, K, 2 * x_rows, p.bn))
+      return CLLM_EINVAL;
+    maps[i].a1 = maps[i].a2 = maps[i].a0;
+  }
+  std::vector<void*> tmp;
+  auto alloc = [&](size_t bytes) -> void* {
+    void* v = nullptr;
+    if (cudaMalloc(&v, bytes) != cudaSuccess || cudaMemset(v, 0, bytes) != cudaSuccess) return nullptr;
+    tmp.push_back(v);
+    return v;
+  };
+  int rc = CLLM_OK;
+  cudaStream_t s = nullptr;
+  cudaGraph_t graph = nullptr;
+  cudaGraphExec_t exec = nullptr;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  do {
+    float* part = static_cast<float*>(alloc(static_cast<size_t>(mtiles) * p.maxc * p.bn * kBM * 4));
+    int* tickets = static_cast<int*>(alloc(mtiles * 4));
+    int* err = static_cast<int*>(alloc(16));
+    float* ssq = static_cast<float*>(alloc(static_cast<size_t>(mtiles) * ldt * 4));
+    void* xg = alloc(static_cast<size_t>(T) * M * 2 * 2);
+    void* ones = alloc(static_cast<size_t>(M) * 2);
+    if (!part || !tickets || !err || !ssq || !xg || !ones) {
+      rc = CLLM_ENOMEM;
+      break;
+    }
+    if (cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreate(&e0) != cudaSuccess || cudaEventCreate(&e1) != cudaSuccess) {
+      rc = CLLM_ECUDA;
+      break;
+    }
+    GemmArgs g{};
+    g.M = M;
+    g.K = K;
+    g.T = T;
+    g.mtiles = p.mtiles;
+    g.ntiles = p.ntiles;
+    g.kchunks = p.kchunks;
+    g.cpc = p.cpc;
+    g.bn = p.bn;
+    g.maxc = p.maxc;
+    g.rows_q = M;
+    g.rows_qk = M;
+    g.lo_rows = x_rows;
+    g.l2_ahead = l2_ahead;
+    g.partial = part;
+    g.tickets = tickets;
+    g.err = err;
+    EpiArgs e{};
+    e.T = T;
+    e.ldt = ldt;
+    e.x = Y;
+    e.xg = xg;
+    e.gnext = ones;
+    e.plane_x = static_cast<size_t>(T) * M;
+    e.ssq_out = ssq;
+    e.d = M;
+    e.err = err;
+    if (cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) != cudaSuccess) {
+      rc = CLLM_ECUDA;
+      break;
+    }
+    cudaError_t le = cudaSuccess;
+    for (int i = 0; i < iters && le == cudaSuccess; ++i)
+      le = launch_gemm_tc(EPI_RESID, p.bn_max, maps[i % n_w], g, e, p.grid, s, pdl != 0);
+    cudaError_t ce = cudaStreamEndCapture(s, &graph);
+    if (le != cudaSuccess || ce != cudaSuccess ||
+        cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess) {
+      rc = CLLM_ECUDA;
+      break;
+    }
+    if (cudaGraphLaunch(exec, s) != cudaSuccess || cudaEventRecord(e0, s) != cudaSuccess ||
+        cudaGraphLaunch(exec, s) != cudaSuccess || cudaEventRecord(e1, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess) {
+      rc = CLLM_ECUDA;
+      break;
+    }
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, e0, e1);
+    *us_per_launch = ms * 1000.f / iters;
+    int herr = 0;
+    cudaMemcpy(&herr, err, 4, cudaMemcpyDeviceToHost);
+    if (herr) rc = (herr & DERR_TIMEOUT) ? CLLM_ETIMEOUT : CLLM_EDEVICE;
+  } while (0);
+  if (exec) cudaGraphExecDestroy(exec);
+  if (graph) cudaGraphDestroy(graph);
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  if (s) cudaStreamDestroy(s);
   for (void* v : tmp) cudaFree(v);
   return rc;
 }

@@ -256,16 +256,25 @@ __device__ void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
 // ---------------------------------------------------------------------------------
 
 // Stage = one 128 x 64 weight tile + the hi and lo planes of a BNMAX x 64
-// activation tile.  Up to BNMAX = 64 two CTAs fit on an SM (so the next
-// kernel's CTAs can start while this one drains).
+// activation tile.  One CTA per SM with as many stages as fit: the weight
+// stream is latency-bound by the bytes in flight per SM (~45 GB/s per SM at
+// ~1.8 us loaded DRAM latency needs > 80 KB in flight).
 template <int BNMAX>
 struct TcCfg {
-  static constexpr int STAGES = BNMAX <= 32 ? 4 : (BNMAX <= 64 ? 3 : (BNMAX <= 128 ? 3 : 2));
+  static constexpr int STAGES = BNMAX <= 32 ? 8 : (BNMAX <= 64 ? 6 : (BNMAX <= 128 ? 4 : 2));
   static constexpr int A_BYTES = kBM * kBK * 2;
   static constexpr int B_HALF = BNMAX * kBK * 2;
   static constexpr int B_BYTES = 2 * B_HALF;
+  // The hi and lo products land in separate accumulator columns and are summed
+  // in the epilogue, for every BNMAX, so a token's result is the same
+  // whatever the launch's token count.  BNMAX <= 128: the lo rows follow the
+  // bn hi rows in shared memory and one MMA with N = 2*bn covers both (lo at
+  // column bn + t); BNMAX = 256: two MMAs, lo into columns 256 + t.
+  static constexpr bool STACKED = BNMAX <= 128;
+  static constexpr int ACC_COLS = 2 * BNMAX;
+  static constexpr int NACC = ACC_COLS <= 256 ? 2 : 1;  // accumulators in TMEM (512 columns)
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int TMEM_COLS = 2 * BNMAX;  // two accumulators: 64, 128, 256 or 512
+  static constexpr int TMEM_COLS = NACC * ACC_COLS;  // 128, 256, 512 or 512
   static constexpr size_t BAR_BYTES = 8 * (2 * STAGES + 5) + 16;
   static constexpr size_t SMEM =
       1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + sizeof(EpiSmem) + 16 + BAR_BYTES;
@@ -275,9 +284,6 @@ struct Segment {
   int unit, k0, k1;
 };
 
-// Weight tiles per CTA prefetched into L2 ahead of the shared-memory ring
-// (16 x 16 KB x 152 CTAs ~ 40 MB of the 129 MB L2).
-constexpr int kL2Ahead = 16;
 
 // Iterate the (unit, k-range) segments of the chunk range [c, c1).
 __device__ __forceinline__ bool next_segment(int& c, int c1, int kchunks, Segment& sg) {
@@ -387,17 +393,18 @@ __global__ void __launch_bounds__(192, 1)
         const int row0 = tile_mode ? nt * BNMAX : 0;
         uint8_t* dst = sB + st * Cfg::B_BYTES;
         tma_load_2d(dst, &mB, &full[st], k * kBK, row0, pol_x);
-        tma_load_2d(dst + Cfg::B_HALF, &mB, &full[st], k * kBK, g.lo_rows + row0, pol_x);
+        tma_load_2d(dst + (Cfg::STACKED ? g.bn * kBK * 2 : Cfg::B_HALF), &mB, &full[st], k * kBK,
+                    g.lo_rows + row0, pol_x);
       };
       // Weights do not depend on earlier kernels: start streaming them before
       // waiting for the previous kernel (programmatic dependent launch) --
-      // the first S tiles into shared memory, the next kL2Ahead into L2.
+      // the first S tiles into shared memory, the next g.l2_ahead into L2.
       const int pre = min(S, nchunks);
       for (int idx = 0; idx < pre; ++idx) {
         mbar_arrive_expect_tx(&full[idx], Cfg::A_BYTES + b_bytes);
         load_a(idx);
       }
-      for (int idx = pre; idx < min(nchunks, pre + kL2Ahead); ++idx) {
+      for (int idx = pre; idx < min(nchunks, pre + g.l2_ahead); ++idx) {
         const int c = c0 + idx;
         const int u = unit_of(c), k = c - u * g.kchunks;
         const int mt = u / g.ntiles;
@@ -437,7 +444,7 @@ __global__ void __launch_bounds__(192, 1)
   } else if (warp == 1) {
     if (lane == 0 && c0 < c1) {
       // ---------------- MMA issuer ----------------
-      const uint32_t idesc = idesc_bf16_f32(kBM, g.bn);
+      const uint32_t idesc = idesc_bf16_f32(kBM, Cfg::STACKED ? 2 * g.bn : g.bn);
       int c = c0, idx = 0, acc = 0;
       uint32_t accph = 0;
       Segment sg;
@@ -445,7 +452,7 @@ __global__ void __launch_bounds__(192, 1)
       while (ok && next_segment(c, c1, g.kchunks, sg)) {
         if (!mbar_wait(&tempty[acc], accph ^ 1, abort_flag)) break;
         tc_fence_after();
-        const uint32_t dt = tmem + static_cast<uint32_t>(acc * BNMAX);
+        const uint32_t dt = tmem + static_cast<uint32_t>(acc * Cfg::ACC_COLS);
         for (int k = sg.k0; k < sg.k1; ++k, ++idx) {
           const int st = idx % S;
           if (!mbar_wait(&full[st], (idx / S) & 1, abort_flag)) {
@@ -460,14 +467,18 @@ __global__ void __launch_bounds__(192, 1)
             const uint64_t ad = sdesc_kmajor_sw128(a_addr + kk * 32);
             tc_mma_f16(dt, ad, sdesc_kmajor_sw128(b_addr + kk * 32), idesc,
                        (k > sg.k0 || kk > 0) ? 1u : 0u);
-            tc_mma_f16(dt, ad, sdesc_kmajor_sw128(b_addr + Cfg::B_HALF + kk * 32), idesc, 1u);
+            if (!Cfg::STACKED)
+              tc_mma_f16(dt + BNMAX, ad, sdesc_kmajor_sw128(b_addr + Cfg::B_HALF + kk * 32), idesc,
+                         (k > sg.k0 || kk > 0) ? 1u : 0u);
           }
           tc_commit(&empty[st]);
         }
         if (!ok) break;
         tc_commit(&tfull[acc]);
-        acc ^= 1;
-        if (acc == 0) accph ^= 1;
+        if (++acc == Cfg::NACC) {
+          acc = 0;
+          accph ^= 1;
+        }
       }
       // Every issued MMA has completed before TMEM is released.
       tc_commit(drain);
@@ -498,11 +509,17 @@ __global__ void __launch_bounds__(192, 1)
       const int ncols = min(g.bn, e.T - tbase);
       const int nchunk = (ncols + kEpiCols - 1) / kEpiCols;
       const uint32_t taddr =
-          tmem + (static_cast<uint32_t>(grp * 32) << 16) + static_cast<uint32_t>(acc * BNMAX);
+          tmem + (static_cast<uint32_t>(grp * 32) << 16) + static_cast<uint32_t>(acc * Cfg::ACC_COLS);
       float* mypart = g.partial + (static_cast<size_t>(u) * g.maxc + slot) * g.bn * kBM;
       for (int ch = 0; ch < nchunk; ++ch) {
         float v[kEpiCols];
         tmem_ld16(taddr + ch * kEpiCols, v);
+        {
+          float vlo[kEpiCols];
+          tmem_ld16(taddr + (Cfg::STACKED ? g.bn : BNMAX) + ch * kEpiCols, vlo);
+#pragma unroll
+          for (int j = 0; j < kEpiCols; ++j) v[j] += vlo[j];
+        }
         if (nc == 1) {
           epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es);
         } else {
@@ -542,8 +559,10 @@ __global__ void __launch_bounds__(192, 1)
       } else if (KIND == EPI_ARGMAX) {
         epi_argmax_finish(e, r, es);
       }
-      acc ^= 1;
-      if (acc == 0) accph ^= 1;
+      if (++acc == Cfg::NACC) {
+        acc = 0;
+        accph ^= 1;
+      }
     }
   }
   tc_fence_before();

@@ -71,6 +71,7 @@ struct GemmArgs {
   int mtiles, ntiles, kchunks, cpc, bn, maxc;
   int rows_q, rows_qk;  // QKV: first rows of the K and V sections (weight-map select)
   int lo_rows;          // row offset of the activations' lo plane in the B map
+  int l2_ahead;         // weight tiles per CTA prefetched into L2 before the PDL wait
   float* partial;       // [units*maxc][bn][128] split-K partial tiles
   int* tickets;         // [units] arrival counters (self-resetting)
   // SIMT (fp32) path only
