@@ -1,0 +1,239 @@
+// Fused epilogues of the weight-streaming GEMMs (shared by the per-GEMM kernels
+// and the persistent per-iteration kernel).
+//   EPI_QKV    : x rms-scale, rotate-half RoPE, Q -> scratch, K/V -> cache
+//   EPI_GATEUP : x rms-scale, silu(gate) * up -> h
+//   EPI_RESID  : residual add into the fp32 stream, next norm's input and
+//                per-tile sum of squares
+//   EPI_ARGMAX : x rms-scale, per-tile (max, argmax, 2nd max) of the logits;
+//                the last tile to finish reduces them to argmax and top-2 gap
+#pragma once
+#include <float.h>
+#include <limits.h>
+
+#include "act.cuh"
+#include "internal.cuh"
+#include "ptx.cuh"
+
+namespace cllm {
+
+// ---------------------------------------------------------------------------------
+// Epilogues.  128 threads; thread r owns weight row r of the tile and 16
+// consecutive token columns t0..t0+15.  Named barrier 1 syncs the 128 threads.
+// ---------------------------------------------------------------------------------
+
+struct EpiSmem {
+  float x[kEpiCols][kBM + 1];
+  float rs[kEpiCols];
+  float red[4][kEpiCols];
+  float am[4][kEpiCols][3];
+  int flag;
+  int ok;
+};
+
+__device__ __forceinline__ void epi_sync() { named_bar_sync(1, 128); }
+
+__device__ __forceinline__ void epi_norm_scale(const EpiArgs& e, int t0, int r, EpiSmem& s) {
+  if (r < kEpiCols) {
+    const int t = t0 + r;
+    float rs = 0.f;
+    if (t < e.T) {
+      float acc = 0.f;
+      for (int i = 0; i < e.ssq_tiles; ++i) acc += e.ssq_in[static_cast<size_t>(i) * e.ldt + t];
+      rs = rsqrtf(acc * e.inv_d + e.eps);
+    }
+    s.rs[r] = rs;
+  }
+  epi_sync();
+}
+
+// (max, argmax with lowest index on ties, second max) merge
+__device__ __forceinline__ void am_merge(float& v1, int& i1, float& v2, float w1, int j1, float w2) {
+  const bool other_hi = (w1 > v1) || (w1 == v1 && j1 < i1);
+  if (other_hi) {
+    v2 = fmaxf(w2, v1);
+    v1 = w1;
+    i1 = j1;
+  } else {
+    v2 = fmaxf(v2, w1);
+  }
+}
+
+template <int KIND, typename Act>
+__device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols], int r,
+                          EpiSmem& s) {
+  const int lane = r & 31, grp = r >> 5;
+  if (KIND == EPI_QKV) {
+    epi_norm_scale(e, t0, r, s);
+    const int m = mt * kBM + r;
+    const int sec = (m < e.dq) ? 0 : (m < e.dq + e.dkv ? 1 : 2);  // uniform over the tile
+    const int ms = m - (sec == 0 ? 0 : (sec == 1 ? e.dq : e.dq + e.dkv));
+    const int head = ms / e.hd, i = ms - head * e.hd, half = e.hd >> 1;
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) v[j] *= s.rs[j];
+    if (sec < 2) {
+#pragma unroll
+      for (int j = 0; j < kEpiCols; ++j) s.x[j][r] = v[j];
+      epi_sync();
+      const int rp = (i < half) ? r + half : r - half;
+      const int fi = (i < half) ? i : i - half;
+#pragma unroll
+      for (int j = 0; j < kEpiCols; ++j) {
+        const int t = t0 + j;
+        if (t < e.T) {
+          const int p = min(e.pos[t], e.max_seq - 1);
+          const float2 cs = e.rope[static_cast<size_t>(p) * half + fi];
+          const float pv = s.x[j][rp];
+          v[j] = (i < half) ? (v[j] * cs.x - pv * cs.y) : (v[j] * cs.x + pv * cs.y);
+        }
+      }
+      epi_sync();
+    }
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      const int t = t0 + j;
+      if (t >= e.T) continue;
+      using AT = typename AttnType<Act>::T;
+      if (sec == 0) {
+        st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
+      } else {
+        const int p = e.pos[t], b = e.bidx[t];
+        if (p < 0 || p >= e.max_seq) {
+          atomicOr(e.err, DERR_CAPACITY);
+          continue;
+        }
+        const size_t off =
+            ((static_cast<size_t>(b) * e.n_kv_heads + head) * e.max_seq + p) * e.hd + i;
+        st_act(reinterpret_cast<AT*>(sec == 1 ? e.k_cache : e.v_cache), off, v[j]);
+      }
+    }
+  } else if (KIND == EPI_GATEUP) {
+    epi_norm_scale(e, t0, r, s);
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      v[j] *= s.rs[j];
+      s.x[j][r] = v[j];
+    }
+    epi_sync();
+    if (r < 64) {
+      const int f = mt * 64 + r;
+      if (f < e.F) {
+#pragma unroll
+        for (int j = 0; j < kEpiCols; ++j) {
+          const int t = t0 + j;
+          if (t < e.T) {
+            const float gt = v[j], up = s.x[j][r + 64];
+            st_gin(reinterpret_cast<Act*>(e.h_out), static_cast<size_t>(t) * e.F + f, e.plane_h,
+                   gt / (1.f + expf(-gt)) * up);
+          }
+        }
+      }
+    }
+    epi_sync();
+  } else if (KIND == EPI_RESID) {
+    const int m = mt * kBM + r;
+    const float gn = ld_act(reinterpret_cast<const Act*>(e.gnext), m);
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      const int t = t0 + j;
+      float sq = 0.f;
+      if (t < e.T) {
+        const size_t o = static_cast<size_t>(t) * e.d + m;
+        const float xi = e.x[o] + v[j];
+        e.x[o] = xi;
+        st_gin(reinterpret_cast<Act*>(e.xg), o, e.plane_x, xi * gn);
+        sq = xi * xi;
+      }
+      sq = warp_sum(sq);
+      if (lane == 0) s.red[grp][j] = sq;
+    }
+    epi_sync();
+    if (r < kEpiCols) {
+      const int t = t0 + r;
+      if (t < e.T)
+        e.ssq_out[static_cast<size_t>(mt) * e.ldt + t] =
+            ((s.red[0][r] + s.red[1][r]) + s.red[2][r]) + s.red[3][r];
+    }
+    epi_sync();
+  } else {  // EPI_ARGMAX
+    epi_norm_scale(e, t0, r, s);
+    const int m = mt * kBM + r;
+    const bool vrow = m < e.V;
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      const int t = t0 + j;
+      const float lg = v[j] * s.rs[j];
+      if (e.logits != nullptr && t < e.T && vrow) e.logits[static_cast<size_t>(t) * e.V + m] = lg;
+      float v1 = vrow ? lg : -INFINITY, v2 = -INFINITY;
+      int i1 = m;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float w1 = __shfl_xor_sync(0xffffffffu, v1, o);
+        const int j1 = __shfl_xor_sync(0xffffffffu, i1, o);
+        const float w2 = __shfl_xor_sync(0xffffffffu, v2, o);
+        am_merge(v1, i1, v2, w1, j1, w2);
+      }
+      if (lane == 0) {
+        s.am[grp][j][0] = v1;
+        s.am[grp][j][1] = __int_as_float(i1);
+        s.am[grp][j][2] = v2;
+      }
+    }
+    epi_sync();
+    if (r < kEpiCols) {
+      const int t = t0 + r;
+      if (t < e.T) {
+        float v1 = s.am[0][r][0], v2 = s.am[0][r][2];
+        int i1 = __float_as_int(s.am[0][r][1]);
+        for (int gq = 1; gq < 4; ++gq)
+          am_merge(v1, i1, v2, s.am[gq][r][0], __float_as_int(s.am[gq][r][1]), s.am[gq][r][2]);
+        float* dst = e.am_part + (static_cast<size_t>(mt) * e.ldt + t) * 3;
+        dst[0] = v1;
+        dst[1] = __int_as_float(i1);
+        dst[2] = v2;
+      }
+    }
+    epi_sync();
+  }
+}
+
+// After a unit's argmax partials are written: the last unit of the launch to
+// finish reduces all tiles to pred[t] (argmax, lowest index on ties) and
+// gap[t] = top1 - top2.  The merge is exact, so the order does not matter.
+__device__ void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
+  __threadfence();
+  epi_sync();
+  if (r == 0) {
+    const int old = atomicAdd(e.am_ticket, 1);
+    s.flag = (old == e.am_units - 1);
+  }
+  epi_sync();
+  const bool last = s.flag;
+  epi_sync();
+  if (!last) return;
+  __threadfence();
+  for (int tb = 0; tb < e.T; tb += 16) {
+    const int t = tb + (r >> 3), part = r & 7;
+    float v1 = -INFINITY, v2 = -INFINITY;
+    int i1 = INT_MAX;
+    if (t < e.T) {
+      for (int mt = part; mt < e.am_mtiles; mt += 8) {
+        const float* p = e.am_part + (static_cast<size_t>(mt) * e.ldt + t) * 3;
+        am_merge(v1, i1, v2, __ldcg(p), __float_as_int(__ldcg(p + 1)), __ldcg(p + 2));
+      }
+    }
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+      const float w1 = __shfl_xor_sync(0xffffffffu, v1, o);
+      const int j1 = __shfl_xor_sync(0xffffffffu, i1, o);
+      const float w2 = __shfl_xor_sync(0xffffffffu, v2, o);
+      am_merge(v1, i1, v2, w1, j1, w2);
+    }
+    if (part == 0 && t < e.T) {
+      e.pred[t] = i1;
+      e.gap[t] = v1 - v2;
+    }
+  }
+  if (r == 0) *e.am_ticket = 0;
+}
+
+}  // namespace cllm
