@@ -174,6 +174,10 @@ int cllm_ar_decode(cllm_ctx *ctx, int B, const int32_t *tokens, const int32_t *l
 /* Static description of a status code. */
 const char *cllm_status_string(int status);
 
+/* The last CUDA call that made a call of this thread return CLLM_ECUDA
+ * ("<where>: <cudaError name>"), or "none". */
+const char *cllm_last_cuda_error(void);
+
 /* ---- device-resident decode loop ---------------------------------------------
  * The three calls cllm_jacobi_decode is made of, for callers that time or
  * drive the loop themselves (inputs and state stay in device memory).
@@ -194,13 +198,39 @@ int cllm_decode_run(cllm_ctx *ctx, int max_iters, int *iters_run, int64_t *commi
  * per-sequence iteration counts [B] (either may be NULL). */
 int cllm_decode_read(cllm_ctx *ctx, int32_t *tokens_out, int32_t *iters_out);
 
+/* ---- options --------------------------------------------------------------------
+ * CLLM_OPT_PERSISTENT (default 1): run each decode/step iteration of the bf16
+ * engine as ONE persistent kernel (one CTA per SM; phases embed, per layer
+ * QKV / attention / O / gate-up / down, LM head, accept, separated by grid
+ * barriers) when B*n <= 128 and head_dim is 64 or 128; 0 = one kernel per
+ * phase.  Both paths compute bit-identical results.  Takes effect for graphs
+ * captured after the call.  Returns CLLM_OK or EINVAL (unknown option).
+ */
+#define CLLM_OPT_PERSISTENT 1
+/* CLLM_OPT_PRE_STAGES (default: the whole ring): in the persistent kernel,
+ * weight tiles per CTA issued for the next GEMM phase before its grid barrier
+ * opens. */
+#define CLLM_OPT_PRE_STAGES 3
+/* CLLM_OPT_L2_AHEAD (default 0): in the persistent kernel, weight tiles
+ * (16 KB each) per CTA that the TMA producer prefetches into L2 for the next
+ * GEMM phase once its shared-memory ring is full, while the previous phase
+ * drains.  0..4096. */
+#define CLLM_OPT_L2_AHEAD 2
+int cllm_set_option(cllm_ctx *ctx, int option, int value);
+
+/* 1 if an iteration of width n on the current batch runs as the persistent
+ * kernel, 0 if as one kernel per phase, or a negative status. */
+int cllm_uses_persistent(cllm_ctx *ctx, int n);
+
 /* ---- introspection ----------------------------------------------------------- */
 
 /* Per-launch device time of each kernel class in the last profiled iteration
  * (cllm_set_profiling(ctx, 1) captures CUDA events around every kernel of the
  * iteration graph).  names/ms: up to cap entries; returns the entry count.
  * Kernel classes: "embed", "gemm_qkv", "attention", "attn_combine", "gemm_o",
- * "gemm_gateup", "gemm_down", "gemm_lmhead", "accept". */
+ * "gemm_gateup", "gemm_down", "gemm_lmhead", "accept"; for the persistent
+ * kernel: "step_persistent" (the kernel) and "phase:<class>" (per-phase time
+ * from in-kernel timestamps of CTA 0). */
 int cllm_set_profiling(cllm_ctx *ctx, int on);
 int cllm_profile_read(cllm_ctx *ctx, const char **names, float *ms_total, int *launches,
                       int cap);

@@ -40,6 +40,23 @@ int cllm_test_gemm_bf16_timed(const void *W, long long w_stride_bytes, int n_w, 
                               float *Y, int M, int K, int T, int x_rows, int iters, int pdl,
                               int l2_ahead, float *us_per_launch);
 
+/*
+ * Raw phase timestamps (globaltimer ns) of the last profiled iteration of the
+ * persistent kernel (cllm_set_profiling(ctx, 1)): out[0..P] CTA 0's phase
+ * starts and end; then, per phase p, out[P+1+p] first and out[2P+1+p] last
+ * start over the CTAs, out[3P+1+p] first and out[4P+1+p] last arrival at the
+ * grid barrier.  names[p] = phase class.  Returns the number of values (5P+1),
+ * 0 if nothing was profiled.
+ */
+int cllm_test_phase_stamps(cllm_ctx *ctx, unsigned long long *out, int cap, const char **names,
+                           int names_cap);
+
+/* Per-CTA timestamps of the last profiled persistent iteration:
+ * out[(k * P + p) * G + cta], k = 0 phase start (dependency seen), 1 MMA
+ * issuer done with the phase (GEMM phases), 2 arrival at the grid barrier;
+ * G = SM count.  Returns the number of values (3 * P * G). */
+int cllm_test_cta_stamps(cllm_ctx *ctx, unsigned long long *out, long long cap);
+
 #ifdef __cplusplus
 }
 #endif

@@ -26,7 +26,11 @@ CLLM_BLOCK_REFILL = 0
 EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode",
            "cllm_ar_decode", "cllm_status_string", "cllm_decode_begin", "cllm_decode_run",
            "cllm_decode_read", "cllm_set_profiling", "cllm_profile_read",
-           "cllm_kernels_per_iteration", "cllm_committed_lengths", "cllm_gemm_bf16_noalloc")
+           "cllm_kernels_per_iteration", "cllm_committed_lengths", "cllm_gemm_bf16_noalloc",
+           "cllm_set_option", "cllm_uses_persistent", "cllm_last_cuda_error")
+CLLM_OPT_PERSISTENT = 1
+CLLM_OPT_L2_AHEAD = 2
+CLLM_OPT_PRE_STAGES = 3
 
 
 class CllmError(RuntimeError):
@@ -102,6 +106,12 @@ def load(build_if_missing: bool = True):
     lib.cllm_gemm_bf16_noalloc.argtypes = [vp, vp, vp, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                            ctypes.c_int, vp]
     lib.cllm_gemm_bf16_noalloc.restype = ctypes.c_int
+    lib.cllm_set_option.argtypes = [vp, ctypes.c_int, ctypes.c_int]
+    lib.cllm_set_option.restype = ctypes.c_int
+    lib.cllm_uses_persistent.argtypes = [vp, ctypes.c_int]
+    lib.cllm_uses_persistent.restype = ctypes.c_int
+    lib.cllm_last_cuda_error.argtypes = []
+    lib.cllm_last_cuda_error.restype = ctypes.c_char_p
     for name in ("cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode", "cllm_ar_decode",
                  "cllm_decode_begin", "cllm_decode_run", "cllm_decode_read", "cllm_set_profiling",
                  "cllm_profile_read", "cllm_kernels_per_iteration", "cllm_committed_lengths"):
@@ -119,6 +129,11 @@ def _status_string(s: int) -> str:
 
 def _check(rc: int, where: str):
     if rc != CLLM_OK:
+        if rc == -3:
+            try:
+                where += " [" + load(build_if_missing=False).cllm_last_cuda_error().decode() + "]"
+            except Exception:
+                pass
         raise CllmError(rc, where)
 
 
@@ -248,6 +263,21 @@ class Engine:
         its = np.zeros(self.B, dtype=np.int32)
         _check(self._lib.cllm_decode_read(self._h, _ip(out), _ip(its)), "cllm_decode_read")
         return out, its
+
+    def set_persistent(self, on: bool):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PERSISTENT, 1 if on else 0), "cllm_set_option")
+
+    def set_l2_ahead(self, tiles: int):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_L2_AHEAD, int(tiles)), "cllm_set_option")
+
+    def set_pre_stages(self, tiles: int):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PRE_STAGES, int(tiles)), "cllm_set_option")
+
+    def uses_persistent(self, n: int) -> bool:
+        r = self._lib.cllm_uses_persistent(self._h, n)
+        if r < 0:
+            raise CllmError(r, "cllm_uses_persistent")
+        return bool(r)
 
     def set_profiling(self, on: bool):
         _check(self._lib.cllm_set_profiling(self._h, 1 if on else 0), "cllm_set_profiling")

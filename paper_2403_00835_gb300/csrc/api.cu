@@ -10,6 +10,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <memory>
 #include <new>
 #include <string>
 #include <tuple>
@@ -152,7 +153,8 @@ struct cllm_ctx {
       *iters = nullptr, *done = nullptr, *out = nullptr, *accepted = nullptr, *prompts = nullptr,
       *plen = nullptr, *status = nullptr, *err = nullptr;
   size_t out_cap = 0;
-  int* status_host = nullptr;  // pinned: {active, committed, device error}
+  int* status_host = nullptr;  // pinned: slots of 4 ints {active, committed, device error, -}
+  cudaEvent_t iter_ev[2] = {nullptr, nullptr};
   // host state
   int B = 0;
   std::vector<int> lens, Lh;
@@ -165,8 +167,22 @@ struct cllm_ctx {
     cudaGraphExec_t exec = nullptr;
     int2* qtiles = nullptr;
     int launches = 0;
+    bool persistent = false;
+    int n_phases = 0;
+    std::vector<int> phase_kind;       // PhaseKind / EPI_* per phase (profiling)
+    std::vector<std::string> phase_names;
+    std::vector<void*> bufs;           // device tables owned by the graph
+    unsigned long long* stamps = nullptr;
+    unsigned long long* cta_stamps = nullptr;
   };
-  std::map<std::tuple<int, int, int, int, int, unsigned long long, int, int>, GraphEntry> graphs;
+  bool persistent = true;  // one persistent kernel per iteration where supported
+  int l2_ahead_persistent = 0;  // weight tiles per CTA prefetched into L2 at a barrier
+  int pre_stages = 1 << 20;     // weight tiles issued before a phase's barrier opens
+  std::vector<unsigned long long> last_stamps;  // last profiled persistent iteration
+  std::vector<std::string> last_phase_names;
+  std::vector<unsigned long long> last_cta_stamps;
+  std::map<std::tuple<int, int, int, int, int, unsigned long long, int, int, int, int>, GraphEntry>
+      graphs;
   // profiling
   bool profiling = false;
   std::vector<cudaEvent_t> prof_events;
@@ -179,6 +195,13 @@ struct cllm_ctx {
 
 namespace {
 
+thread_local char g_last_cuda_error[160] = "none";
+
+// Record a failed CUDA call (name and where) and return CLLM_ECUDA.
+int cuda_fail(cudaError_t e, const char* where) {
+  snprintf(g_last_cuda_error, sizeof g_last_cuda_error, "%s: %s", where, cudaGetErrorName(e));
+  return CLLM_ECUDA;
+}
 
 template <typename T>
 bool dev_alloc(cllm_ctx* c, T** p, size_t bytes) {
@@ -230,6 +253,33 @@ EpiArgs base_epi(cllm_ctx* c, int T) {
   return e;
 }
 
+// Work split and epilogue bookkeeping of one bf16 GEMM of T tokens.
+GemmArgs tc_gemm_args(cllm_ctx* c, int mtiles, int M, int K, int T, EpiArgs& e, Part* part) {
+  GemmArgs g{};
+  g.M = M;
+  g.K = K;
+  g.T = T;
+  g.rows_q = c->dq;
+  g.rows_qk = c->dq + c->dkv;
+  g.err = c->err;
+  g.tickets = c->tickets;
+  g.partial = c->gemm_part;
+  g.lo_rows = c->Tcap;
+  g.l2_ahead = kL2AheadDefault;
+  g.pre_stages = 1 << 20;
+  const Part p = plan_gemm(mtiles, K, T, c->sms);
+  g.mtiles = p.mtiles;
+  g.ntiles = p.ntiles;
+  g.kchunks = p.kchunks;
+  g.cpc = p.cpc;
+  g.bn = p.bn;
+  g.maxc = p.maxc;
+  e.am_units = mtiles * p.ntiles;
+  e.am_mtiles = mtiles;
+  if (part) *part = p;
+  return g;
+}
+
 // One GEMM launch: D[m][t] = W[m] . X[t] with epilogue `kind`.
 cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, int M, int K, int T,
                  const void* X, const void* A0, const void* A1, const void* A2,
@@ -246,6 +296,7 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
   g.partial = c->gemm_part;
   g.lo_rows = c->Tcap;
   g.l2_ahead = kL2AheadDefault;
+  g.pre_stages = 1 << 20;
   cudaError_t err;
   if (!c->bf16) {
     g.mtiles = mtiles;
@@ -260,13 +311,9 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
     ee.am_mtiles = mtiles;
     err = launch_gemm_simt(kind, g, ee, s, pdl);
   } else {
-    const Part p = plan_gemm(mtiles, K, T, c->sms);
-    g.mtiles = p.mtiles;
-    g.ntiles = p.ntiles;
-    g.kchunks = p.kchunks;
-    g.cpc = p.cpc;
-    g.bn = p.bn;
-    g.maxc = p.maxc;
+    EpiArgs ee = e;
+    Part p;
+    g = tc_gemm_args(c, mtiles, M, K, T, ee, &p);
     if (static_cast<size_t>(mtiles) * p.maxc * p.bn * kBM > c->gemm_part_elems && p.ntiles == 1)
       return cudaErrorInvalidValue;
     GemmMaps maps{};
@@ -276,9 +323,6 @@ cudaError_t gemm(cllm_ctx* c, cudaStream_t s, bool pdl, int kind, int mtiles, in
     if (!make_map(&maps.b, X, static_cast<uint64_t>(K), static_cast<uint64_t>(2 * c->Tcap),
                   static_cast<uint32_t>(p.bn)))
       return cudaErrorInvalidValue;
-    EpiArgs ee = e;
-    ee.am_units = mtiles * p.ntiles;
-    ee.am_mtiles = mtiles;
     err = launch_gemm_tc(kind, p.bn_max, maps, g, ee, p.grid, s, pdl);
   }
   return after_launch(c, s, name, err);
@@ -296,12 +340,8 @@ struct FwdSpec {
   AcceptArgs acc;  // step/decode
 };
 
-// Issue one forward (+ accept) on stream s.
-cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool pdl) {
-  cudaError_t err;
+EmbedArgs make_embed_args(cllm_ctx* c, const FwdSpec& f) {
   const int T = f.T;
-  const int ab = c->bf16 ? 1 : 0;
-  // embedding
   EmbedArgs ea{};
   ea.emb = c->tok_emb;
   ea.gain = c->layers[0].attn_norm;
@@ -330,8 +370,11 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
   ea.seq_row0 = c->seq_row0;
   ea.seq_nrows = c->seq_nrows;
   ea.err = c->err;
-  if ((err = after_launch(c, s, "embed", launch_embed(ea, ab, s, pdl))) != cudaSuccess) return err;
+  return ea;
+}
 
+AttnArgs make_attn_args(cllm_ctx* c, const FwdSpec& f) {
+  const int T = f.T;
   AttnArgs aa{};
   aa.q = c->q;
   aa.seq_start = c->seq_start;
@@ -352,6 +395,17 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
   aa.plane_out = c->planes == 2 ? static_cast<size_t>(c->Tcap) * c->dq : 0;
   aa.T = T;
   aa.err = c->err;
+  return aa;
+}
+
+// Issue one forward (+ accept) on stream s.
+cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool pdl) {
+  cudaError_t err;
+  const int T = f.T;
+  const int ab = c->bf16 ? 1 : 0;
+  const EmbedArgs ea = make_embed_args(c, f);
+  if ((err = after_launch(c, s, "embed", launch_embed(ea, ab, s, pdl))) != cudaSuccess) return err;
+  AttnArgs aa = make_attn_args(c, f);
 
   for (int l = 0; l < c->NL; ++l) {
     const LayerW& L = c->layers[l];
@@ -464,10 +518,11 @@ AcceptArgs make_accept(cllm_ctx* c, int B, int n, bool decode) {
 // Read the device status (active, committed, error) after a synchronisation.
 int check_device_error(cllm_ctx* c) {
   int e = 0;
-  if (cudaMemcpyAsync(&c->status_host[2], c->err, sizeof(int), cudaMemcpyDeviceToHost,
-                      c->stream) != cudaSuccess)
-    return CLLM_ECUDA;
-  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return CLLM_ECUDA;
+  cudaError_t ce = cudaMemcpyAsync(&c->status_host[2], c->err, sizeof(int), cudaMemcpyDeviceToHost,
+                                   c->stream);
+  if (ce != cudaSuccess) return cuda_fail(ce, "status copy");
+  ce = cudaStreamSynchronize(c->stream);
+  if (ce != cudaSuccess) return cuda_fail(ce, "stream sync");
   e = c->status_host[2];
   if (e == 0) return CLLM_OK;
   cudaMemsetAsync(c->err, 0, sizeof(int), c->stream);
@@ -489,13 +544,185 @@ int attn_grid_for(cllm_ctx* c, int n_qtiles) {
   return static_cast<int>(std::max(1L, std::min(items, 2L * c->sms)));
 }
 
+
+// Tables of the persistent per-iteration kernel for B sequences x n rows:
+// tensor maps [7 per layer: q k v o gate up down][LM head][xg, attn, h] and
+// the phases [embed][per layer: QKV, attention, O, gate/up, down][LM head][accept].
+int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, int n_qtiles,
+                     cllm_ctx::GraphEntry& ge, StepParams& prm, int& bn_max) {
+  StepArgs& sa = prm.a;
+  const int T = B * n;
+  const int NL = c->NL;
+  const int mapB = 7 * NL + 1;
+  std::vector<CUtensorMap> maps(7 * NL + 4);
+  for (int l = 0; l < NL; ++l) {
+    const LayerW& L = c->layers[l];
+    maps[7 * l + 0] = L.mq;
+    maps[7 * l + 1] = L.mk;
+    maps[7 * l + 2] = L.mv;
+    maps[7 * l + 3] = L.mo;
+    maps[7 * l + 4] = L.mgate;
+    maps[7 * l + 5] = L.mup;
+    maps[7 * l + 6] = L.mdown;
+  }
+  maps[7 * NL] = c->mlm;
+  const uint32_t bn = static_cast<uint32_t>(round_up(T, 16));
+  const uint64_t rows = 2 * static_cast<uint64_t>(c->Tcap);
+  if (!make_map(&maps[mapB], c->xg, c->d, rows, bn) ||
+      !make_map(&maps[mapB + 1], c->attn, c->dq, rows, bn) ||
+      !make_map(&maps[mapB + 2], c->h, c->F, rows, bn))
+    return CLLM_EINVAL;
+
+  FwdSpec f{};
+  f.mode = mode;
+  f.T = T;
+  f.B = B;
+  f.n = n;
+  f.qtiles = qtiles;
+  f.n_qtiles = n_qtiles;
+  std::vector<PhaseDesc> ph;
+  auto gemm_phase = [&](int epi, int m0, int m1, int m2, int mb, int mtiles, int M, int K,
+                        EpiArgs e) {
+    PhaseDesc d{};
+    d.kind = PH_GEMM;
+    d.epi = epi;
+    d.map_a0 = m0;
+    d.map_a1 = m1;
+    d.map_a2 = m2;
+    d.map_b = mb;
+    Part p;
+    d.g = tc_gemm_args(c, mtiles, M, K, T, e, &p);
+    d.g.l2_ahead = c->l2_ahead_persistent;
+    d.g.pre_stages = c->pre_stages;
+    d.e = e;
+    bn_max = p.bn_max;
+    ph.push_back(d);
+  };
+  {
+    PhaseDesc d{};
+    d.kind = PH_EMBED;
+    ph.push_back(d);
+  }
+  const int Mqkv = c->dq + 2 * c->dkv;
+  for (int l = 0; l < NL; ++l) {
+    const LayerW& L = c->layers[l];
+    const size_t kvoff = static_cast<size_t>(l) * c->layer_kv_elems * c->esz;
+    void* kl = static_cast<char*>(c->kc) + kvoff;
+    void* vl = static_cast<char*>(c->vc) + kvoff;
+    EpiArgs e = base_epi(c, T);
+    e.ssq_in = c->ssq;
+    e.q_out = c->q;
+    e.k_cache = kl;
+    e.v_cache = vl;
+    gemm_phase(EPI_QKV, 7 * l, 7 * l + 1, 7 * l + 2, mapB, Mqkv / kBM, Mqkv, c->d, e);
+    PhaseDesc at{};
+    at.kind = PH_ATTN;
+    at.k_cache = kl;
+    at.v_cache = vl;
+    ph.push_back(at);
+    e = base_epi(c, T);
+    e.x = c->x;
+    e.xg = c->xg;
+    e.gnext = L.mlp_norm;
+    e.ssq_out = c->ssq;
+    gemm_phase(EPI_RESID, 7 * l + 3, 7 * l + 3, 7 * l + 3, mapB + 1, c->d / kBM, c->d, c->dq, e);
+    e = base_epi(c, T);
+    e.ssq_in = c->ssq;
+    e.h_out = c->h;
+    gemm_phase(EPI_GATEUP, 7 * l + 4, 7 * l + 5, 7 * l + 4, mapB, ceil_div(c->F, 64), c->F, c->d, e);
+    e = base_epi(c, T);
+    e.x = c->x;
+    e.xg = c->xg;
+    e.gnext = (l + 1 < NL) ? c->layers[l + 1].attn_norm : c->final_norm;
+    e.ssq_out = c->ssq;
+    gemm_phase(EPI_RESID, 7 * l + 6, 7 * l + 6, 7 * l + 6, mapB + 2, c->d / kBM, c->d, c->F, e);
+  }
+  {
+    EpiArgs e = base_epi(c, T);
+    e.am_part = c->am_part;
+    e.am_ticket = c->am_ticket;
+    e.pred = c->pred;
+    e.gap = c->gap;
+    e.logits = nullptr;
+    e.ssq_in = c->ssq;
+    gemm_phase(EPI_ARGMAX, 7 * NL, 7 * NL, 7 * NL, mapB, ceil_div(c->V, kBM), c->V, c->d, e);
+    PhaseDesc d{};
+    d.kind = PH_ACCEPT;
+    ph.push_back(d);
+  }
+  ge.phase_kind.clear();
+  ge.phase_names.clear();
+  int resid_seen = 0;
+  for (const PhaseDesc& d : ph) {
+    ge.phase_kind.push_back(d.kind == PH_GEMM ? 10 + d.epi : d.kind);
+    const char* nm = "accept";
+    if (d.kind == PH_EMBED) nm = "embed";
+    else if (d.kind == PH_ATTN) nm = "attention";
+    else if (d.kind == PH_GEMM && d.epi == EPI_QKV) nm = "gemm_qkv";
+    else if (d.kind == PH_GEMM && d.epi == EPI_GATEUP) nm = "gemm_gateup";
+    else if (d.kind == PH_GEMM && d.epi == EPI_ARGMAX) nm = "gemm_lmhead";
+    else if (d.kind == PH_GEMM && d.epi == EPI_RESID) nm = (resid_seen++ % 2 == 0) ? "gemm_o" : "gemm_down";
+    ge.phase_names.push_back(nm);
+  }
+  // device copies
+  auto upload = [&](const void* src, size_t bytes) -> void* {
+    void* p = nullptr;
+    if (cudaMalloc(&p, bytes) != cudaSuccess) return nullptr;
+    ge.bufs.push_back(p);
+    if (src && cudaMemcpy(p, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess) return nullptr;
+    if (!src && cudaMemset(p, 0, bytes) != cudaSuccess) return nullptr;
+    return p;
+  };
+  if (maps.size() > static_cast<size_t>(kMaxStepMaps)) return CLLM_EUNSUPPORTED;
+  for (size_t i = 0; i < maps.size(); ++i) prm.maps[i] = maps[i];
+  void* ph_d = upload(ph.data(), ph.size() * sizeof(PhaseDesc));
+  void* tk_d = upload(nullptr, static_cast<size_t>(n_qtiles) * c->H * sizeof(int) + 16);
+  void* bar_d = upload(nullptr, 64);
+  void* st_d = upload(nullptr, (5 * ph.size() + 1) * sizeof(unsigned long long));
+  void* cst_d = upload(nullptr, 6 * ph.size() * c->sms * sizeof(unsigned long long));
+  if (!ph_d || !tk_d || !bar_d || !st_d || !cst_d) return CLLM_ENOMEM;
+  ge.cta_stamps = static_cast<unsigned long long*>(cst_d);
+  if (c->profiling) {
+    // epilogue stamps k = 3..5 of the per-CTA stamp array
+    const long long PG = static_cast<long long>(ph.size()) * c->sms;
+    for (size_t p = 0; p < ph.size(); ++p)
+      if (ph[p].kind == PH_GEMM) {
+        ph[p].e.dbg = ge.cta_stamps + 3 * PG + static_cast<long long>(p) * c->sms;
+        ph[p].e.dbg_stride = PG;
+      }
+    if (cudaMemcpy(ph_d, ph.data(), ph.size() * sizeof(PhaseDesc), cudaMemcpyHostToDevice) !=
+        cudaSuccess)
+      return CLLM_ECUDA;
+  }
+  ge.n_phases = static_cast<int>(ph.size());
+  ge.stamps = static_cast<unsigned long long*>(st_d);
+  sa = StepArgs{};
+  sa.phases = static_cast<const PhaseDesc*>(ph_d);
+  sa.n_phases = ge.n_phases;
+  sa.bar = static_cast<unsigned*>(bar_d);
+  sa.embed = make_embed_args(c, f);
+  sa.attn = make_attn_args(c, f);
+  sa.attn_tickets = static_cast<int*>(tk_d);
+  sa.accept = make_accept(c, B, n, mode == MODE_DECODE);
+  sa.stamps = c->profiling ? ge.stamps : nullptr;
+  sa.cta_stamps = c->profiling ? ge.cta_stamps : nullptr;
+  sa.err = c->err;
+  return CLLM_OK;
+}
+
+bool persistent_ok(cllm_ctx* c, int B, int n) {
+  return c->bf16 && c->persistent && B * n <= 128 && 7 * c->NL + 4 <= kMaxStepMaps &&
+         B * ceil_div(n, kQTile) <= kMaxQTilesStep && (c->hd == 64 || c->hd == 128);
+}
+
 // Get (capturing on first use) the graph of one decode/step iteration.
 int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
   const int B = c->B;
   auto key = std::make_tuple(mode, B, n, mode == MODE_DECODE ? c->dec_max_new : 0,
                              mode == MODE_DECODE ? c->dec_opts.eos_id : 0,
                              mode == MODE_DECODE ? static_cast<unsigned long long>(c->dec_opts.seed) : 0ull,
-                             mode == MODE_DECODE ? c->dec_opts.guess_init : 0, c->profiling ? 1 : 0);
+                             mode == MODE_DECODE ? c->dec_opts.guess_init : 0, c->profiling ? 1 : 0,
+                             c->persistent ? 1 : 0, c->l2_ahead_persistent * 65536 + std::min(c->pre_stages, 65535));
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
     *out = &it->second;
@@ -508,6 +735,103 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
       cudaSuccess) {
     cudaFree(ge.qtiles);
     return CLLM_ECUDA;
+  }
+  if (persistent_ok(c, B, n)) {
+    std::unique_ptr<StepParams> prm(new (std::nothrow) StepParams());
+    if (!prm) return CLLM_ENOMEM;
+    StepArgs& sa = prm->a;
+    int bn_max = 32;
+    int rc = build_persistent(c, mode, B, n, ge.qtiles, static_cast<int>(qt.size()), ge, *prm, bn_max);
+    if (rc != CLLM_OK) {
+      cudaFree(ge.qtiles);
+      for (void* p : ge.bufs) cudaFree(p);
+      return rc;
+    }
+    ge.persistent = true;
+    const bool prof = c->profiling;
+    if (prof) {
+      while (c->prof_events.size() < 2) {
+        cudaEvent_t ev;
+        if (cudaEventCreate(&ev) != cudaSuccess) return CLLM_ECUDA;
+        c->prof_events.push_back(ev);
+      }
+    }
+    cudaGraph_t g = nullptr;
+    cudaError_t e = cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal);
+    if (e != cudaSuccess) return cuda_fail(e, "begin capture (persistent)");
+    e = cudaMemsetAsync(sa.bar, 0, 64, c->stream);
+    if (e == cudaSuccess && prof) {
+      // first-of slots start at all-ones (atomicMin), last-of slots at zero
+      const size_t P = ge.n_phases;
+      e = cudaMemsetAsync(ge.stamps + P + 1, 0xff, 2 * P * 8, c->stream);
+      if (e == cudaSuccess) e = cudaMemsetAsync(ge.stamps + P + 1 + P, 0, P * 8, c->stream);
+      if (e == cudaSuccess) e = cudaMemsetAsync(ge.stamps + P + 1 + 2 * P, 0xff, P * 8, c->stream);
+      if (e == cudaSuccess) e = cudaMemsetAsync(ge.stamps + P + 1 + 3 * P, 0, P * 8, c->stream);
+    }
+    if (e == cudaSuccess && prof)
+      e = cudaEventRecordWithFlags(c->prof_events[0], c->stream, cudaEventRecordExternal);
+    if (e == cudaSuccess) {
+      e = launch_step_persistent(*prm, bn_max, c->hd, c->sms, c->stream, false);
+    }
+    const cudaError_t first = e;
+    if (e == cudaSuccess && prof)
+      e = cudaEventRecordWithFlags(c->prof_events[1], c->stream, cudaEventRecordExternal);
+    cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
+    if (e != cudaSuccess || e2 != cudaSuccess) {
+      if (g) cudaGraphDestroy(g);
+      cudaFree(ge.qtiles);
+      for (void* p : ge.bufs) cudaFree(p);
+      return first != cudaSuccess ? cuda_fail(first, "capture of the persistent iteration")
+                                  : cuda_fail(e2, "end capture (persistent)");
+    }
+    ge.launches = 1;
+    {  // mark the kernel node cooperative where the driver supports it
+      size_t nn = 0;
+      if (cudaGraphGetNodes(g, nullptr, &nn) == cudaSuccess && nn > 0) {
+        std::vector<cudaGraphNode_t> nodes(nn);
+        if (cudaGraphGetNodes(g, nodes.data(), &nn) == cudaSuccess) {
+          for (auto nd : nodes) {
+            cudaGraphNodeType ty;
+            if (cudaGraphNodeGetType(nd, &ty) == cudaSuccess && ty == cudaGraphNodeTypeKernel) {
+              cudaLaunchAttributeValue v{};
+              v.cooperative = 1;
+              if (cudaGraphKernelNodeSetAttribute(nd, cudaLaunchAttributeCooperative, &v) !=
+                  cudaSuccess)
+                cudaGetLastError();
+            }
+          }
+        }
+      }
+    }
+    e = cudaGraphInstantiate(&ge.exec, g, 0);
+    if (e != cudaSuccess) {
+      // without the cooperative attribute (co-residency by construction)
+      cudaGetLastError();
+      size_t nn = 0;
+      std::vector<cudaGraphNode_t> nodes;
+      if (cudaGraphGetNodes(g, nullptr, &nn) == cudaSuccess) {
+        nodes.resize(nn);
+        cudaGraphGetNodes(g, nodes.data(), &nn);
+        for (auto nd : nodes) {
+          cudaGraphNodeType ty;
+          if (cudaGraphNodeGetType(nd, &ty) == cudaSuccess && ty == cudaGraphNodeTypeKernel) {
+            cudaLaunchAttributeValue v{};
+            v.cooperative = 0;
+            cudaGraphKernelNodeSetAttribute(nd, cudaLaunchAttributeCooperative, &v);
+          }
+        }
+      }
+      e = cudaGraphInstantiate(&ge.exec, g, 0);
+    }
+    cudaGraphDestroy(g);
+    if (e != cudaSuccess) {
+      cudaFree(ge.qtiles);
+      for (void* p : ge.bufs) cudaFree(p);
+      return cuda_fail(e, "instantiate (persistent)");
+    }
+    auto res = c->graphs.emplace(key, ge);
+    *out = &res.first->second;
+    return CLLM_OK;
   }
   FwdSpec f{};
   f.mode = mode;
@@ -540,11 +864,6 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
   cudaError_t e = cudaSuccess;
   if (prof) e = cudaEventRecordWithFlags(c->prof_events[0], c->stream, cudaEventRecordExternal);
   if (e == cudaSuccess) e = record_forward(c, c->stream, f, !prof);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(c->status_host, c->status, 2 * sizeof(int), cudaMemcpyDeviceToHost,
-                        c->stream);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(&c->status_host[2], c->err, sizeof(int), cudaMemcpyDeviceToHost, c->stream);
   cudaError_t e2 = cudaStreamEndCapture(c->stream, &g);
   c->rec_names = nullptr;
   if (e != cudaSuccess || e2 != cudaSuccess) {
@@ -565,7 +884,31 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
   return CLLM_OK;
 }
 
-void accumulate_profile(cllm_ctx* c) {
+void accumulate_profile(cllm_ctx* c, const cllm_ctx::GraphEntry* ge) {
+  if (ge && ge->persistent) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, c->prof_events[0], c->prof_events[1]) == cudaSuccess) {
+      auto& a = c->prof_acc["step_persistent"];
+      a.first += ms;
+      a.second += 1;
+    }
+    std::vector<unsigned long long> st(5 * ge->n_phases + 1);
+    if (cudaMemcpy(st.data(), ge->stamps, st.size() * 8, cudaMemcpyDeviceToHost) != cudaSuccess)
+      return;
+    c->last_stamps = st;
+    c->last_phase_names = ge->phase_names;
+    c->last_cta_stamps.resize(6 * static_cast<size_t>(ge->n_phases) * c->sms);
+    cudaMemcpy(c->last_cta_stamps.data(), ge->cta_stamps, c->last_cta_stamps.size() * 8,
+               cudaMemcpyDeviceToHost);
+    // phase p runs from CTA 0 seeing its dependency met to the next phase's
+    for (int p = 0; p < ge->n_phases; ++p) {
+      if (st[p + 1] < st[p] || st[p] == 0) continue;
+      auto& a = c->prof_acc["phase:" + ge->phase_names[p]];
+      a.first += (st[p + 1] - st[p]) * 1e-6;
+      a.second += 1;
+    }
+    return;
+  }
   for (size_t i = 0; i < c->prof_names.size() && i + 1 < c->prof_events.size(); ++i) {
     float ms = 0.f;
     if (cudaEventElapsedTime(&ms, c->prof_events[i], c->prof_events[i + 1]) == cudaSuccess) {
@@ -576,8 +919,8 @@ void accumulate_profile(cllm_ctx* c) {
   }
 }
 
-int read_status(cllm_ctx* c) {
-  const int e = c->status_host[2];
+int read_status(cllm_ctx* c, int slot) {
+  const int e = c->status_host[4 * slot + 2];
   if (e == 0) return CLLM_OK;
   cudaMemsetAsync(c->err, 0, sizeof(int), c->stream);
   cudaStreamSynchronize(c->stream);
@@ -591,6 +934,8 @@ int read_status(cllm_ctx* c) {
 // =====================================================================================
 // C ABI
 // =====================================================================================
+
+extern "C" const char* cllm_last_cuda_error(void) { return g_last_cuda_error; }
 
 extern "C" const char* cllm_status_string(int s) {
   switch (s) {
@@ -614,10 +959,13 @@ extern "C" void cllm_destroy(cllm_ctx* c) {
   for (auto& kv : c->graphs) {
     if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
     if (kv.second.qtiles) cudaFree(kv.second.qtiles);
+    for (void* p : kv.second.bufs) cudaFree(p);
   }
   for (auto ev : c->prof_events) cudaEventDestroy(ev);
   for (void* p : c->allocs) cudaFree(p);
   if (c->status_host) cudaFreeHost(c->status_host);
+  for (auto ev : c->iter_ev)
+    if (ev) cudaEventDestroy(ev);
   if (c->own_stream && c->stream) cudaStreamDestroy(c->stream);
   delete c;
 }
@@ -716,7 +1064,8 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
         rc = CLLM_EINVAL;
         break;
       }
-      if (gemm_tc_set_attributes() != cudaSuccess || attention_set_attributes() != cudaSuccess) {
+      if (gemm_tc_set_attributes() != cudaSuccess || attention_set_attributes() != cudaSuccess ||
+          step_persistent_set_attributes() != cudaSuccess) {
         rc = CLLM_ECUDA;
         break;
       }
@@ -803,11 +1152,16 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
       rc = CLLM_ENOMEM;
       break;
     }
-    if (cudaMallocHost(&c->status_host, 16) != cudaSuccess) {
+    if (cudaMallocHost(&c->status_host, 32) != cudaSuccess) {
       rc = CLLM_ENOMEM;
       break;
     }
-    std::memset(c->status_host, 0, 16);
+    std::memset(c->status_host, 0, 32);
+    if (cudaEventCreateWithFlags(&c->iter_ev[0], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&c->iter_ev[1], cudaEventDisableTiming) != cudaSuccess) {
+      rc = CLLM_ECUDA;
+      break;
+    }
     if (cudaDeviceSynchronize() != cudaSuccess) {
       rc = CLLM_ECUDA;
       break;
@@ -978,7 +1332,8 @@ extern "C" int cllm_jacobi_step(cllm_ctx* c, const int32_t* guess, int n, int32_
     int rc = get_graph(c, MODE_STEP, n, &ge);
     c->profiling = prof;
     if (rc != CLLM_OK) return rc;
-    if (cudaGraphLaunch(ge->exec, c->stream) != cudaSuccess) return CLLM_ECUDA;
+    cudaError_t e = cudaGraphLaunch(ge->exec, c->stream);
+    if (e != cudaSuccess) return cuda_fail(e, "graph launch (step)");
   }
   std::vector<int> acc(B);
   if (cudaMemcpyAsync(next_out, c->pred, static_cast<size_t>(B) * n * 4, cudaMemcpyDeviceToHost,
@@ -1026,6 +1381,7 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
     for (auto& kv : c->graphs) {
       if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
       if (kv.second.qtiles) cudaFree(kv.second.qtiles);
+      for (void* p : kv.second.bufs) cudaFree(p);
     }
     c->graphs.clear();
   }
@@ -1049,18 +1405,59 @@ extern "C" int cllm_decode_run(cllm_ctx* c, int max_iters, int* iters_run, int64
   cllm_ctx::GraphEntry* ge = nullptr;
   int rc = get_graph(c, MODE_DECODE, c->dec_n, &ge);
   if (rc != CLLM_OK) return rc;
+  // Iteration j+1 is queued before iteration j's 12-byte status is read, so
+  // the device never waits for the host; once no sequence is active the
+  // queued iteration commits nothing.  (Profiling reads per-iteration timing
+  // and runs one iteration at a time.)
+  auto issue = [&](int j) -> cudaError_t {
+    const int slot = j & 1;
+    cudaError_t e = cudaGraphLaunch(ge->exec, c->stream);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(&c->status_host[4 * slot], c->status, 2 * sizeof(int),
+                          cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(&c->status_host[4 * slot + 2], c->err, sizeof(int),
+                          cudaMemcpyDeviceToHost, c->stream);
+    if (e == cudaSuccess) e = cudaEventRecord(c->iter_ev[slot], c->stream);
+    return e;
+  };
+  const bool pipelined = !c->profiling;
   int it = 0;
   int64_t com = 0;
-  for (; it < max_iters;) {
-    if (cudaGraphLaunch(ge->exec, c->stream) != cudaSuccess) return CLLM_ECUDA;
-    if (cudaStreamSynchronize(c->stream) != cudaSuccess) return CLLM_ECUDA;
-    ++it;
-    if (c->profiling) accumulate_profile(c);
-    rc = read_status(c);
-    if (rc != CLLM_OK) return rc;
-    com += c->status_host[1];
-    if (c->status_host[0] == 0) break;
+  int queued = 0;  // iterations issued
+  cudaError_t e = cudaSuccess;
+  if (max_iters > 0) {
+    e = issue(0);
+    if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+    queued = 1;
   }
+  while (it < max_iters) {
+    if (pipelined && queued < max_iters && queued == it + 1) {
+      e = issue(queued);
+      if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+      ++queued;
+    }
+    e = cudaEventSynchronize(c->iter_ev[it & 1]);
+    if (e != cudaSuccess) return cuda_fail(e, "iteration sync");
+    if (c->profiling) accumulate_profile(c, ge);
+    const int slot = it & 1;
+    ++it;
+    rc = read_status(c, slot);
+    if (rc != CLLM_OK) {
+      cudaStreamSynchronize(c->stream);
+      return rc;
+    }
+    com += c->status_host[4 * slot + 1];
+    if (c->status_host[4 * slot] == 0) break;
+    if (!pipelined && it < max_iters) {
+      e = issue(it);
+      if (e != cudaSuccess) return cuda_fail(e, "graph launch");
+      ++queued;
+    }
+  }
+  // a queued iteration past the end committed nothing; let it finish
+  e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(e, "stream sync");
   if (iters_run) *iters_run = it;
   if (committed) *committed = com;
   return CLLM_OK;
@@ -1106,6 +1503,30 @@ extern "C" int cllm_ar_decode(cllm_ctx* c, int B, const int32_t* tokens, const i
   o.guess_init = CLLM_GUESS_UNIFORM;
   o.block_mode = CLLM_BLOCK_REFILL;
   return cllm_jacobi_decode(c, B, tokens, lens, 1, max_new, &o, tokens_out, nullptr);
+}
+
+extern "C" int cllm_set_option(cllm_ctx* c, int option, int value) {
+  if (!c) return CLLM_EINVAL;
+  if (option == CLLM_OPT_PERSISTENT) {
+    c->persistent = value != 0;
+    return CLLM_OK;
+  }
+  if (option == CLLM_OPT_PRE_STAGES) {
+    if (value < 0) return CLLM_EINVAL;
+    c->pre_stages = value;
+    return CLLM_OK;
+  }
+  if (option == CLLM_OPT_L2_AHEAD) {
+    if (value < 0 || value > 4096) return CLLM_EINVAL;
+    c->l2_ahead_persistent = value;
+    return CLLM_OK;
+  }
+  return CLLM_EINVAL;
+}
+
+extern "C" int cllm_uses_persistent(cllm_ctx* c, int n) {
+  if (!c || !c->prefilled) return CLLM_EINVAL;
+  return persistent_ok(c, c->B, n) ? 1 : 0;
 }
 
 extern "C" int cllm_set_profiling(cllm_ctx* c, int on) {
@@ -1215,6 +1636,7 @@ extern "C" int cllm_test_gemm_bf16(const void* W, const void* X, float* Y, int M
     g.rows_qk = M;
     g.lo_rows = x_rows;
     g.l2_ahead = kL2AheadDefault;
+    g.pre_stages = 1 << 20;
     g.partial = part;
     g.tickets = tickets;
     g.err = err;
@@ -1309,6 +1731,7 @@ extern "C" int cllm_test_gemm_bf16_timed(const void* W, long long w_stride_bytes
     g.rows_qk = M;
     g.lo_rows = x_rows;
     g.l2_ahead = l2_ahead;
+    g.pre_stages = 1 << 20;
     g.partial = part;
     g.tickets = tickets;
     g.err = err;
@@ -1355,4 +1778,21 @@ extern "C" int cllm_test_gemm_bf16_timed(const void* W, long long w_stride_bytes
   if (s) cudaStreamDestroy(s);
   for (void* v : tmp) cudaFree(v);
   return rc;
+}
+
+extern "C" int cllm_test_phase_stamps(cllm_ctx* c, unsigned long long* out, int cap,
+                                      const char** names, int names_cap) {
+  if (!c) return CLLM_EINVAL;
+  const int n = static_cast<int>(c->last_stamps.size());
+  for (int i = 0; i < n && i < cap; ++i) out[i] = c->last_stamps[i];
+  for (int i = 0; i < static_cast<int>(c->last_phase_names.size()) && i < names_cap; ++i)
+    names[i] = c->last_phase_names[i].c_str();
+  return n;
+}
+
+extern "C" int cllm_test_cta_stamps(cllm_ctx* c, unsigned long long* out, long long cap) {
+  if (!c) return CLLM_EINVAL;
+  const long long n = static_cast<long long>(c->last_cta_stamps.size());
+  for (long long i = 0; i < n && i < cap; ++i) out[i] = c->last_cta_stamps[i];
+  return static_cast<int>(n);
 }

@@ -1,0 +1,334 @@
+// One work item of the block attention (16-row query tile x head x 128-key
+// chunk) on tensor cores, and the merge of a query tile's chunk partials.
+// Shared by the attention kernel (a CTA of 128 threads) and the persistent
+// per-iteration kernel (its four epilogue warps); `sync` is the barrier of
+// those 128 threads and `tid` their index 0..127.
+#pragma once
+#include "act.cuh"
+#include "internal.cuh"
+#include "ptx.cuh"
+
+namespace cllm {
+
+template <int HD>
+struct AttnTileSmem {
+  __half q[kQTile][HD + 8];
+  __half k[kAttnChunk][HD + 8];  // reused as float co[4][kQTile][HD] for the warp merge
+  __half v[kAttnChunk][HD + 8];
+  float m[4][kQTile];
+  float l[4][kQTile];
+};
+
+// Where the iteration's query-tile and sequence metadata are read from: the
+// kernel arguments (global memory), or a shared-memory copy made once per
+// phase (AttnMetaSmem) so that work items do not chain dependent loads.
+struct GlobalMeta {
+  const AttnArgs& a;
+  __device__ int2 qtile(int q) const { return a.qtiles[q]; }
+  __device__ int start(int b) const { return a.seq_start[b]; }
+  __device__ int row0(int b) const { return a.seq_row0[b]; }
+  __device__ int nrows(int b) const { return a.seq_nrows[b]; }
+};
+
+constexpr int kMetaMaxBatch = 128;
+
+struct AttnMetaSmem {
+  int2 qt[kMaxQTilesStep];
+  int start[kMetaMaxBatch];
+  int row0[kMetaMaxBatch];
+  int nrows[kMetaMaxBatch];
+};
+
+struct SmemMeta {
+  const AttnMetaSmem& m;
+  __device__ int2 qtile(int q) const { return m.qt[q]; }
+  __device__ int start(int b) const { return m.start[b]; }
+  __device__ int row0(int b) const { return m.row0[b]; }
+  __device__ int nrows(int b) const { return m.nrows[b]; }
+};
+
+// Copy the metadata of `a` into shared memory (128 threads, one round trip).
+__device__ __forceinline__ void attn_meta_load(const AttnArgs& a, AttnMetaSmem& m, int tid, int B) {
+  for (int q = tid; q < a.n_qtiles; q += 128) m.qt[q] = a.qtiles[q];
+  for (int b = tid; b < B; b += 128) {
+    m.start[b] = __ldcg(a.seq_start + b);
+    m.row0[b] = __ldcg(a.seq_row0 + b);
+    m.nrows[b] = __ldcg(a.seq_nrows + b);
+  }
+}
+
+// Number of key chunks the query tile qi reaches (its last row's position).
+template <class Meta>
+__device__ __forceinline__ int attn_tile_chunks(const AttnArgs& a, const Meta& md, int qi) {
+  const int2 qt = md.qtile(qi);
+  const int nr = min(kQTile, md.nrows(qt.x) - qt.y);
+  if (nr <= 0) return 0;
+  const int pos_last = md.start(qt.x) + qt.y + nr - 1;
+  return min(pos_last / kAttnChunk + 1, a.nch_max);
+}
+__device__ __forceinline__ int attn_tile_chunks(const AttnArgs& a, int qi) {
+  return attn_tile_chunks(a, GlobalMeta{a}, qi);
+}
+
+// Prefix sum of work items over query tiles into pre[0..n_qtiles];
+// items(q) = H * chunks(q).  Warp 0 of the group scans; returns the total.
+template <class Sync, class Meta = GlobalMeta>
+__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync, const Meta& md) {
+  if (tid < 32) {
+    int carry = 0;
+    for (int base = 0; base < a.n_qtiles; base += 32) {
+      const int q = base + tid;
+      const int cnt = q < a.n_qtiles ? a.H * attn_tile_chunks(a, md, q) : 0;
+      int incl = cnt;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (tid >= o) incl += y;
+      }
+      if (q < a.n_qtiles) pre[q] = carry + incl - cnt;
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (tid == 0) pre[a.n_qtiles] = carry;
+  }
+  sync();
+  return pre[a.n_qtiles];
+}
+template <class Sync>
+__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync) {
+  return attn_item_prefix(a, pre, tid, sync, GlobalMeta{a});
+}
+
+__device__ __forceinline__ int attn_find_qtile(const int* pre, int n, int item) {
+  int lo = 0, hi = n - 1;  // largest q with pre[q] <= item
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (pre[mid] <= item) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+// Work item `item`: writes the unnormalised chunk partial (O, m, l) of the
+// tile's rows for one head.  Returns the tile index and head in qi_out, h_out.
+template <int HD, class Sync, class Meta = GlobalMeta>
+__device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
+                              int tid, Sync sync, int& qi_out, int& h_out, const Meta& md) {
+  static_assert(sizeof(float) * 4 * kQTile * HD <= sizeof(__half) * kAttnChunk * (HD + 8),
+                "merge area must fit in the K tile");
+  const int warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, cq = lane & 3;
+  const int group = a.H / a.Hkv;
+  const int ldq = a.H * HD;
+  const __half* Q = static_cast<const __half*>(a.q);
+  const __half* KC = static_cast<const __half*>(a.k_cache);
+  const __half* VC = static_cast<const __half*>(a.v_cache);
+  float (*co)[kQTile][HD] = reinterpret_cast<float (*)[kQTile][HD]>(&sm.k[0][0]);
+  const int qi = attn_find_qtile(pre, a.n_qtiles, item);
+  const int local = item - pre[qi];
+  const int c = local / a.H, h = local - c * a.H;
+  const int2 qt = md.qtile(qi);
+  const int b = qt.x, r0 = qt.y;
+  const int nr = min(kQTile, md.nrows(b) - r0);
+  const int start = md.start(b);
+  const int row_g0 = md.row0(b) + r0;
+  const int pos0 = start + r0;  // position of tile row 0
+  const int kb = c * kAttnChunk;
+  int ke = min(kb + kAttnChunk, pos0 + nr);
+  if (ke > a.max_seq) {
+    if (tid == 0) atomicOr(a.err, DERR_CAPACITY);
+    ke = a.max_seq;
+  }
+  const int kvh = h / group;
+  const size_t kvbase = ((static_cast<size_t>(b) * a.Hkv + kvh) * a.max_seq) * HD;
+
+  // ---- stage Q (16 rows), K and V (chunk rows) into shared memory ----
+  constexpr int CPR = HD * 2 / 16;  // 16-byte pieces per row
+  for (int i = tid; i < kQTile * CPR; i += 128) {
+    const int rr = i / CPR, pc = i - rr * CPR;
+    void* dst = &sm.q[rr][pc * 8];
+    if (rr < nr)
+      cp_async16(dst, Q + static_cast<size_t>(row_g0 + rr) * ldq + h * HD + pc * 8);
+    else
+      *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+  }
+  for (int i = tid; i < kAttnChunk * CPR; i += 128) {
+    const int rr = i / CPR, pc = i - rr * CPR;
+    const int key = kb + rr;
+    void* dk = &sm.k[rr][pc * 8];
+    void* dv = &sm.v[rr][pc * 8];
+    if (key < ke) {
+      const size_t off = kvbase + static_cast<size_t>(key) * HD + pc * 8;
+      cp_async16(dk, KC + off);
+      cp_async16(dv, VC + off);
+    } else {
+      *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
+      *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
+    }
+  }
+  cp_async_commit();
+  cp_async_wait_all();
+  sync();
+
+  // ---- per warp: 32 keys x 16 rows ----
+  const int wk0 = warp * 32;  // first key of this warp, relative to kb
+  float o[HD / 8][4];
+#pragma unroll
+  for (int dn = 0; dn < HD / 8; ++dn) o[dn][0] = o[dn][1] = o[dn][2] = o[dn][3] = 0.f;
+  float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
+  if (kb + wk0 < ke) {
+    float s[4][4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ks += 2) {
+      uint32_t qa0[4], qa1[4];
+      ldmatrix_x4(qa0, &sm.q[lane & 15][ks * 16 + (lane >> 4) * 8]);
+      ldmatrix_x4(qa1, &sm.q[lane & 15][(ks + 1) * 16 + (lane >> 4) * 8]);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        uint32_t kb4[4];
+        const int mi = lane >> 3;
+        ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
+        mma_f16_16816(s[j], qa0, kb4[0], kb4[1]);
+        mma_f16_16816(s[j], qa1, kb4[2], kb4[3]);
+      }
+    }
+    // mask + scale (log2 domain)
+    const int posA = pos0 + g, posB = pos0 + g + 8;
+    const bool rowA = g < nr, rowB = g + 8 < nr;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = kb + wk0 + 8 * j + 2 * cq + (e & 1);
+        const bool top = e < 2;
+        const bool valid = key < ke && (top ? (rowA && key <= posA) : (rowB && key <= posB));
+        s[j][e] = valid ? s[j][e] * a.scale_log2 : -INFINITY;
+      }
+      mA = fmaxf(mA, fmaxf(s[j][0], s[j][1]));
+      mB = fmaxf(mB, fmaxf(s[j][2], s[j][3]));
+    }
+    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 1));
+    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 2));
+    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 1));
+    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 2));
+    const float uA = (mA == -INFINITY) ? 0.f : mA;
+    const float uB = (mB == -INFINITY) ? 0.f : mB;
+    uint32_t pa[2][4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float p0 = exp2f(s[j][0] - uA), p1 = exp2f(s[j][1] - uA);
+      const float p2 = exp2f(s[j][2] - uB), p3 = exp2f(s[j][3] - uB);
+      lA += p0 + p1;
+      lB += p2 + p3;
+      pa[j >> 1][(j & 1) * 2 + 0] = pack_f16x2(p0, p1);
+      pa[j >> 1][(j & 1) * 2 + 1] = pack_f16x2(p2, p3);
+    }
+    lA += __shfl_xor_sync(0xffffffffu, lA, 1);
+    lA += __shfl_xor_sync(0xffffffffu, lA, 2);
+    lB += __shfl_xor_sync(0xffffffffu, lB, 1);
+    lB += __shfl_xor_sync(0xffffffffu, lB, 2);
+    // O = P V: A fragments of P for keys 16kk..16kk+15 are the S accumulators
+    // of n-tiles 2kk, 2kk+1 (a0: row g keys 2c.., a1: row g+8, a2/a3: +8 keys).
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+      const uint32_t af[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
+#pragma unroll
+      for (int dn = 0; dn < HD / 8; dn += 2) {
+        uint32_t vb[4];
+        const int mi = lane >> 3;
+        ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
+        mma_f16_16816(o[dn], af, vb[0], vb[1]);
+        mma_f16_16816(o[dn + 1], af, vb[2], vb[3]);
+      }
+    }
+  }
+  sync();  // every warp is done reading K/V before the merge area overwrites K
+#pragma unroll
+  for (int dn = 0; dn < HD / 8; ++dn) {
+    const int d0 = dn * 8 + 2 * cq;
+    co[warp][g][d0] = o[dn][0];
+    co[warp][g][d0 + 1] = o[dn][1];
+    co[warp][g + 8][d0] = o[dn][2];
+    co[warp][g + 8][d0 + 1] = o[dn][3];
+  }
+  if (cq == 0) {
+    sm.m[warp][g] = mA;
+    sm.m[warp][g + 8] = mB;
+    sm.l[warp][g] = lA;
+    sm.l[warp][g + 8] = lB;
+  }
+  sync();
+  {
+    const int row = tid >> 3, part = tid & 7;
+    constexpr int DPT = HD / 8;
+    if (row < nr) {
+      float M = -INFINITY;
+#pragma unroll
+      for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
+      const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + c;
+      float* dst = a.part_o + pidx * HD + part * DPT;
+      if (M == -INFINITY) {
+#pragma unroll
+        for (int dd = 0; dd < DPT; ++dd) dst[dd] = 0.f;
+        if (part == 0) a.part_ml[pidx] = make_float2(-INFINITY, 0.f);
+      } else {
+        float f[4], l = 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+          f[w] = exp2f(sm.m[w][row] - M);
+          l += f[w] * sm.l[w][row];
+        }
+#pragma unroll
+        for (int dd = 0; dd < DPT; ++dd) {
+          const int d = part * DPT + dd;
+          dst[dd] = ((f[0] * co[0][row][d] + f[1] * co[1][row][d]) + f[2] * co[2][row][d]) +
+                    f[3] * co[3][row][d];
+        }
+        if (part == 0) a.part_ml[pidx] = make_float2(M, l);
+      }
+    }
+  }
+  sync();
+  qi_out = qi;
+  h_out = h;
+}
+template <int HD, class Sync>
+__device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
+                              int tid, Sync sync, int& qi_out, int& h_out) {
+  attn_mma_item<HD>(a, item, pre, sm, tid, sync, qi_out, h_out, GlobalMeta{a});
+}
+
+// Merge of the chunk partials 0..pos/128 of every row of query tile qi for
+// head h, in chunk order (the same arithmetic as the attention combine
+// kernel); out = O / l, written as the GEMM input planes.
+template <typename Act, int HD, class Meta>
+__device__ void attn_combine_tile(const AttnArgs& a, int qi, int h, int tid, const Meta& md) {
+  const int2 qt = md.qtile(qi);
+  const int b = qt.x, r0 = qt.y;
+  const int nr = min(kQTile, md.nrows(b) - r0);
+  const int row = tid >> 3, part = tid & 7;
+  constexpr int DPT = HD / 8;
+  if (row >= nr) return;
+  const int t = md.row0(b) + r0 + row;
+  const int pos = md.start(b) + r0 + row;  // the row's position (pos[t])
+  const int nch = min(pos / kAttnChunk + 1, a.nch_max);
+  const size_t base = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
+  float M = -INFINITY;
+  for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&a.part_ml[base + c].x));
+#pragma unroll
+  for (int dd = 0; dd < DPT; ++dd) {
+    const int d = part * DPT + dd;
+    float acc = 0.f, l = 0.f;
+    for (int c = 0; c < nch; ++c) {
+      const float2 ml = __ldcg(&a.part_ml[base + c]);
+      const float f = exp2f(ml.x - M);
+      l += f * ml.y;
+      acc += f * __ldcg(&a.part_o[(base + c) * HD + d]);
+    }
+    st_gin(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * HD + h * HD + d, a.plane_out,
+           acc / l);
+  }
+}
+
+}  // namespace cllm

@@ -21,6 +21,11 @@ namespace cllm {
 // consecutive token columns t0..t0+15.  Named barrier 1 syncs the 128 threads.
 // ---------------------------------------------------------------------------------
 
+// Columns whose per-token epilogue inputs (RMSNorm scale, position, sequence)
+// are prepared once per launch / phase (launches with more tokens prepare them
+// per 16-column chunk).
+constexpr int kEpiPrepMax = 256;
+
 struct EpiSmem {
   float x[kEpiCols][kBM + 1];
   float rs[kEpiCols];
@@ -28,22 +33,86 @@ struct EpiSmem {
   float am[4][kEpiCols][3];
   int flag;
   int ok;
+  int prepared;  // rs_all / pos_all / bidx_all hold this launch's columns
+  float rs_all[kEpiPrepMax];
+  int pos_all[kEpiPrepMax];
+  int bidx_all[kEpiPrepMax];
 };
 
 __device__ __forceinline__ void epi_sync() { named_bar_sync(1, 128); }
 
-__device__ __forceinline__ void epi_norm_scale(const EpiArgs& e, int t0, int r, EpiSmem& s) {
-  if (r < kEpiCols) {
-    const int t = t0 + r;
-    float rs = 0.f;
-    if (t < e.T) {
-      float acc = 0.f;
-      for (int i = 0; i < e.ssq_tiles; ++i) acc += e.ssq_in[static_cast<size_t>(i) * e.ldt + t];
-      rs = rsqrtf(acc * e.inv_d + e.eps);
+// rs[t] = 1 / sqrt(sum of the per-tile sums of squares / d + eps) for the 16
+// columns t0..t0+15: 8 threads per column each sum the tiles i = part (mod 8)
+// in order, then a fixed shuffle tree adds the 8 parts (every load of the
+// column is in flight at once; the order does not depend on the launch).
+// Sum of column t's per-tile squares by the 8 threads part = 0..7 (tiles
+// part, part + 8, ... in order) followed by a fixed shuffle tree.
+__device__ __forceinline__ float epi_ssq_column(const EpiArgs& e, int t, int part, bool valid) {
+  float acc = 0.f;
+  if (valid) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int i = part + 8 * u;
+      v[u] = i < e.ssq_tiles ? __ldcg(e.ssq_in + static_cast<size_t>(i) * e.ldt + t) : 0.f;
     }
-    s.rs[r] = rs;
+#pragma unroll
+    for (int u = 0; u < 8; ++u) acc += v[u];
+    for (int i = part + 64; i < e.ssq_tiles; i += 8) acc += __ldcg(e.ssq_in + static_cast<size_t>(i) * e.ldt + t);
   }
+  acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+  acc += __shfl_xor_sync(0xffffffffu, acc, 2);
+  acc += __shfl_xor_sync(0xffffffffu, acc, 4);
+  return acc;
+}
+
+// Once per launch / phase, before the first accumulator is ready: the RMSNorm
+// scale (kinds that need it), position and sequence index of every column.
+template <int KIND>
+__device__ void epi_prepare(const EpiArgs& e, int r, EpiSmem& s) {
+  s.prepared = 0;
+  if (e.T > kEpiPrepMax) {
+    epi_sync();
+    return;
+  }
+  if (KIND != EPI_RESID) {
+    const int col = r >> 3, part = r & 7;
+    for (int t0 = 0; t0 < e.T; t0 += kEpiCols) {
+      const int t = t0 + col;
+      const float acc = epi_ssq_column(e, t, part, t < e.T);
+      if (part == 0 && t < e.T) s.rs_all[t] = rsqrtf(acc * e.inv_d + e.eps);
+    }
+  }
+  if (KIND == EPI_QKV) {
+    for (int t = r; t < e.T; t += 128) {
+      s.pos_all[t] = e.pos[t];
+      s.bidx_all[t] = e.bidx[t];
+    }
+  }
+  if (r == 0) s.prepared = 1;
   epi_sync();
+}
+
+__device__ __forceinline__ void epi_norm_scale(const EpiArgs& e, int t0, int r, EpiSmem& s) {
+  if (s.prepared) {
+    if (r < kEpiCols) s.rs[r] = (t0 + r < e.T) ? s.rs_all[t0 + r] : 0.f;
+    epi_sync();
+    return;
+  }
+  const int col = r >> 3, part = r & 7;
+  const int t = t0 + col;
+  const float acc = epi_ssq_column(e, t, part, t < e.T);
+  if (part == 0) s.rs[col] = (t < e.T) ? rsqrtf(acc * e.inv_d + e.eps) : 0.f;
+  epi_sync();
+}
+
+// Arrival ticket of the last-arriver pattern: one thread, after a barrier of
+// the 128 epilogue threads; release of the CTA's prior writes (cumulative
+// over the barrier) and acquire of the earlier arrivals' writes.
+__device__ __forceinline__ int ticket_add(int* p, int v) {
+  int old;
+  asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+  return old;
 }
 
 // (max, argmax with lowest index on ties, second max) merge
@@ -58,9 +127,59 @@ __device__ __forceinline__ void am_merge(float& v1, int& i1, float& v2, float w1
   }
 }
 
+// Epilogue inputs that do not depend on the accumulator, loaded before the
+// accumulator / split-K ticket is waited for, so their latency overlaps it:
+// RESID -- the residual stream values and the next norm's gain; QKV -- the
+// RoPE (cos, sin) of each column.  Valid for the 16 columns from t0.
+struct EpiPre {
+  float a[kEpiCols];
+  float b[kEpiCols];
+  float g;
+  int ok;
+  int t0;
+};
+
+template <int KIND, typename Act>
+__device__ __forceinline__ void epi_prefetch(const EpiArgs& e, int mt, int t0, int r,
+                                             const EpiSmem& s, EpiPre& p) {
+  p.ok = 0;
+  p.t0 = t0;
+  if (KIND == EPI_RESID) {
+    const int m = mt * kBM + r;
+    p.g = ld_act(reinterpret_cast<const Act*>(e.gnext), m);
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      const int t = t0 + j;
+      p.a[j] = (t < e.T) ? __ldcg(e.x + static_cast<size_t>(t) * e.d + m) : 0.f;
+    }
+    p.ok = 1;
+  } else if (KIND == EPI_QKV) {
+    if (!s.prepared) return;
+    const int m = mt * kBM + r;
+    const int sec = (m < e.dq) ? 0 : (m < e.dq + e.dkv ? 1 : 2);
+    if (sec == 2) return;
+    const int ms = m - (sec == 0 ? 0 : e.dq);
+    const int i = ms % e.hd, half = e.hd >> 1;
+    const int fi = (i < half) ? i : i - half;
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      const int t = t0 + j;
+      float2 cs = make_float2(1.f, 0.f);
+      if (t < e.T) {
+        const int pp = min(s.pos_all[t], e.max_seq - 1);
+        cs = e.rope[static_cast<size_t>(pp) * half + fi];
+      }
+      p.a[j] = cs.x;
+      p.b[j] = cs.y;
+    }
+    p.ok = 1;
+  }
+}
+
 template <int KIND, typename Act>
 __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols], int r,
-                          EpiSmem& s) {
+                          EpiSmem& s, const EpiPre* pre = nullptr) {
+  const bool use_pre = pre != nullptr && pre->ok && pre->t0 == t0;
   const int lane = r & 31, grp = r >> 5;
   if (KIND == EPI_QKV) {
     epi_norm_scale(e, t0, r, s);
@@ -80,8 +199,13 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
       for (int j = 0; j < kEpiCols; ++j) {
         const int t = t0 + j;
         if (t < e.T) {
-          const int p = min(e.pos[t], e.max_seq - 1);
-          const float2 cs = e.rope[static_cast<size_t>(p) * half + fi];
+          float2 cs;
+          if (use_pre) {
+            cs = make_float2(pre->a[j], pre->b[j]);
+          } else {
+            const int p = min(s.prepared ? s.pos_all[t] : e.pos[t], e.max_seq - 1);
+            cs = e.rope[static_cast<size_t>(p) * half + fi];
+          }
           const float pv = s.x[j][rp];
           v[j] = (i < half) ? (v[j] * cs.x - pv * cs.y) : (v[j] * cs.x + pv * cs.y);
         }
@@ -96,7 +220,8 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
       if (sec == 0) {
         st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
       } else {
-        const int p = e.pos[t], b = e.bidx[t];
+        const int p = s.prepared ? s.pos_all[t] : e.pos[t];
+        const int b = s.prepared ? s.bidx_all[t] : e.bidx[t];
         if (p < 0 || p >= e.max_seq) {
           atomicOr(e.err, DERR_CAPACITY);
           continue;
@@ -131,14 +256,16 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
     epi_sync();
   } else if (KIND == EPI_RESID) {
     const int m = mt * kBM + r;
-    const float gn = ld_act(reinterpret_cast<const Act*>(e.gnext), m);
+    const float gn = use_pre ? pre->g : ld_act(reinterpret_cast<const Act*>(e.gnext), m);
 #pragma unroll
     for (int j = 0; j < kEpiCols; ++j) {
       const int t = t0 + j;
       float sq = 0.f;
       if (t < e.T) {
         const size_t o = static_cast<size_t>(t) * e.d + m;
-        const float xi = e.x[o] + v[j];
+        // L2 read: other CTAs rewrite the residual stream in earlier phases
+        // of the persistent kernel, and L1 is not coherent across SMs
+        const float xi = (use_pre ? pre->a[j] : __ldcg(e.x + o)) + v[j];
         e.x[o] = xi;
         st_gin(reinterpret_cast<Act*>(e.xg), o, e.plane_x, xi * gn);
         sq = xi * xi;
@@ -199,26 +326,40 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
 // After a unit's argmax partials are written: the last unit of the launch to
 // finish reduces all tiles to pred[t] (argmax, lowest index on ties) and
 // gap[t] = top1 - top2.  The merge is exact, so the order does not matter.
-__device__ void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
-  __threadfence();
+__device__ inline void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
   epi_sync();
   if (r == 0) {
-    const int old = atomicAdd(e.am_ticket, 1);
+    const int old = ticket_add(e.am_ticket, 1);
     s.flag = (old == e.am_units - 1);
   }
   epi_sync();
   const bool last = s.flag;
   epi_sync();
   if (!last) return;
-  __threadfence();
   for (int tb = 0; tb < e.T; tb += 16) {
     const int t = tb + (r >> 3), part = r & 7;
     float v1 = -INFINITY, v2 = -INFINITY;
     int i1 = INT_MAX;
     if (t < e.T) {
-      for (int mt = part; mt < e.am_mtiles; mt += 8) {
-        const float* p = e.am_part + (static_cast<size_t>(mt) * e.ldt + t) * 3;
-        am_merge(v1, i1, v2, __ldcg(p), __float_as_int(__ldcg(p + 1)), __ldcg(p + 2));
+      for (int mt0 = part; mt0 < e.am_mtiles; mt0 += 64) {
+        float w1[8], w2[8];
+        int j1[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {  // eight tiles' loads in flight at once
+          const int mt = mt0 + 8 * u;
+          if (mt < e.am_mtiles) {
+            const float* p = e.am_part + (static_cast<size_t>(mt) * e.ldt + t) * 3;
+            w1[u] = __ldcg(p);
+            j1[u] = __float_as_int(__ldcg(p + 1));
+            w2[u] = __ldcg(p + 2);
+          } else {
+            w1[u] = -INFINITY;
+            j1[u] = INT_MAX;
+            w2[u] = -INFINITY;
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) am_merge(v1, i1, v2, w1[u], j1[u], w2[u]);
       }
     }
 #pragma unroll

@@ -159,6 +159,8 @@ __global__ void __launch_bounds__(128) gemm_simt_kernel(const GemmArgs g, const 
     }
     __syncthreads();
   }
+  if (r == 0) es.prepared = 0;
+  __syncthreads();
   epi_apply<KIND, float>(e, mt, t0, acc, r, es);
   if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
 }

@@ -221,13 +221,35 @@ __device__ bool tc_produce(const TcPipe& P, int& idx, int& issued_b, const GemmA
     tma_load_2d(dst + (Cfg::STACKED ? g.bn * kBK * 2 : Cfg::B_HALF), mB, &P.full[st], k * kBK,
                 g.lo_rows + row0, pol_x);
   };
-  // Weight tiles into free stages while the dependency is not satisfied.
+  auto prefetch_l2 = [&](int j) {
+    const int c = c0 + j;
+    const int u = c / g.kchunks, k = c - u * g.kchunks;
+    const int mt = u / g.ntiles;
+    if (KIND == EPI_GATEUP) {
+      tma_prefetch_l2_2d(mA0, k * kBK, mt * 64);
+      tma_prefetch_l2_2d(mA1, k * kBK, mt * 64);
+    } else if (KIND == EPI_QKV) {
+      const int row = mt * kBM;
+      if (row < g.rows_q)
+        tma_prefetch_l2_2d(mA0, k * kBK, row);
+      else if (row < g.rows_qk)
+        tma_prefetch_l2_2d(mA1, k * kBK, row - g.rows_q);
+      else
+        tma_prefetch_l2_2d(mA2, k * kBK, row - g.rows_qk);
+    } else {
+      tma_prefetch_l2_2d(mA0, k * kBK, mt * kBM);
+    }
+  };
+  // Weight tiles into free stages while the dependency is not satisfied; once
+  // the ring is full, the next l2_ahead tiles into L2 (once), so that HBM
+  // keeps streaming while the previous phase drains.
   int j = 0;
   bool open = Dep::kPollable ? dep.ready() : false;
+  bool prefetched = false;
   uint64_t t0 = 0;
   while (j < n && !open) {
     const int gi = idx + j, st = gi % S;
-    if (mbar_try_wait(&P.empty[st], ((gi / S) & 1) ^ 1)) {
+    if (j < g.pre_stages && mbar_try_wait(&P.empty[st], ((gi / S) & 1) ^ 1)) {
       mbar_arrive_expect_tx(&P.full[st], Cfg::A_BYTES + b_bytes);
       load_a(j, st);
       ++j;
@@ -235,6 +257,10 @@ __device__ bool tc_produce(const TcPipe& P, int& idx, int& issued_b, const GemmA
       continue;
     }
     if (!Dep::kPollable) break;
+    if (!prefetched) {
+      for (int jj = j; jj < min(n, j + g.l2_ahead); ++jj) prefetch_l2(jj);
+      prefetched = true;
+    }
     open = dep.ready();
     if (open) break;
     if (*P.abort) return false;
@@ -333,16 +359,21 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
   const int grp = warp & 3;
   const int r = grp * 32 + lane;
   const bool tile_mode = g.ntiles > 1;
+  if (c0 < c1) epi_prepare<KIND>(e, r, es);
   int c = c0;
   Segment sg;
   while (next_segment(c, c1, g.kchunks, sg)) {
     const int u = sg.unit;
     const int mt = u / g.ntiles, nt = u - mt * g.ntiles;
+    EpiPre pre;
+    epi_prefetch<KIND, __nv_bfloat16>(e, mt, tile_mode ? nt * Cfg::BN : 0, r, es, pre);
     if (r == 0) es.ok = mbar_wait(&P.tfull[acc], accph, P.abort) ? 1 : 0;
     epi_sync();
     const bool seg_ok = es.ok != 0;
     epi_sync();
     if (!seg_ok) return false;
+    const bool dbg = e.dbg != nullptr && r == 0 && c >= c1;  // last segment
+    if (dbg) e.dbg[cta] = globaltimer_ns();
     tc_fence_after();
     const int first = (u * g.kchunks) / g.cpc;
     const int last = ((u + 1) * g.kchunks - 1) / g.cpc;
@@ -364,7 +395,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
         for (int j = 0; j < kEpiCols; ++j) v[j] += vlo[j];
       }
       if (nc == 1) {
-        epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es);
+        epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
       } else {
 #pragma unroll
         for (int j = 0; j < kEpiCols; ++j) mypart[(ch * kEpiCols + j) * kBM + r] = v[j];
@@ -374,27 +405,38 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     __syncwarp();
     if (lane == 0) mbar_arrive(&P.tempty[acc]);
     if (nc > 1) {
-      __threadfence();
       epi_sync();
       if (r == 0) {
-        const int old = atomicAdd(&g.tickets[u], 1);
+        const int old = ticket_add(&g.tickets[u], 1);
         es.flag = (old == nc - 1);
       }
       epi_sync();
       const bool last_arrival = es.flag;
       epi_sync();
+      if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
       if (last_arrival) {
-        __threadfence();
         for (int ch = 0; ch < nchunk; ++ch) {
           float v[kEpiCols];
 #pragma unroll
           for (int j = 0; j < kEpiCols; ++j) v[j] = 0.f;
-          for (int s = 0; s < nc; ++s) {
-            const float* p = g.partial + (static_cast<size_t>(u) * g.maxc + s) * g.bn * kBM;
+          // contributors in slot order; each group's loads are issued together
+          for (int s0 = 0; s0 < nc; s0 += 8) {
+            float w[8][kEpiCols];
 #pragma unroll
-            for (int j = 0; j < kEpiCols; ++j) v[j] += __ldcg(p + (ch * kEpiCols + j) * kBM + r);
+            for (int q = 0; q < 8; ++q) {
+              const float* p = g.partial + (static_cast<size_t>(u) * g.maxc + s0 + q) * g.bn * kBM;
+#pragma unroll
+              for (int j = 0; j < kEpiCols; ++j)
+                w[q][j] = (s0 + q < nc) ? __ldcg(p + (ch * kEpiCols + j) * kBM + r) : 0.f;
+            }
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              if (s0 + q < nc) {
+#pragma unroll
+                for (int j = 0; j < kEpiCols; ++j) v[j] += w[q][j];
+              }
           }
-          epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es);
+          epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
         }
         if (r == 0) g.tickets[u] = 0;
         if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
@@ -402,6 +444,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     } else if (KIND == EPI_ARGMAX) {
       epi_argmax_finish(e, r, es);
     }
+    if (dbg) e.dbg[2 * e.dbg_stride + cta] = globaltimer_ns();
     if (++acc == Cfg::NACC) {
       acc = 0;
       accph ^= 1;

@@ -60,6 +60,11 @@ struct EpiArgs {
   float* logits;  // optional debug [T][V]
   int V;
   int* err;
+  // optional timing of the epilogue's last segment (persistent kernel
+  // profiling): dbg[k * dbg_stride + cta], k = 0 accumulator ready, 1 after
+  // the arrival ticket, 2 epilogue done
+  unsigned long long* dbg;
+  long long dbg_stride;
 };
 
 // Work decomposition of one weight-streaming GEMM launch.
@@ -72,6 +77,7 @@ struct GemmArgs {
   int rows_q, rows_qk;  // QKV: first rows of the K and V sections (weight-map select)
   int lo_rows;          // row offset of the activations' lo plane in the B map
   int l2_ahead;         // weight tiles per CTA prefetched into L2 before the PDL wait
+  int pre_stages;       // weight tiles issued before the phase's dependency is met (<= ring)
   float* partial;       // [units*maxc][bn][128] split-K partial tiles
   int* tickets;         // [units] arrival counters (self-resetting)
   // SIMT (fp32) path only
@@ -148,6 +154,51 @@ struct AcceptArgs {
   int prompt_ld;
   int* status;  // [0] active sequences, [1] tokens committed by this iteration
 };
+
+// ---- persistent per-iteration kernel (persistent.cu) ---------------------------------
+
+enum PhaseKind : int { PH_EMBED = 0, PH_GEMM = 1, PH_ATTN = 2, PH_ACCEPT = 3 };
+
+// One phase of an iteration.  GEMM phases name their tensor maps by index
+// into the map table; attention phases carry their layer's K/V cache.
+struct PhaseDesc {
+  int kind, epi;
+  int map_a0, map_a1, map_a2, map_b;
+  GemmArgs g;
+  EpiArgs e;
+  const void* k_cache;
+  const void* v_cache;
+};
+
+struct StepArgs {
+  const PhaseDesc* phases;
+  int n_phases;
+  unsigned* bar;            // grid barrier counter, zero at launch
+  EmbedArgs embed;
+  AttnArgs attn;            // K/V cache set per phase
+  int* attn_tickets;        // [qtiles][heads], self-resetting
+  AcceptArgs accept;
+  unsigned long long* stamps;  // optional: phase start times (CTA 0)
+  unsigned long long* cta_stamps;  // optional: [6][phase][cta] start, MMA done, arrival, epilogue
+  int* err;
+};
+
+constexpr int kMaxQTilesStep = 256;  // query tiles of one iteration (persistent kernel)
+
+// Tensor maps travel by value in the kernel's parameter space (TMA reads
+// descriptors there as it does for per-GEMM kernels): 7 per layer + the LM
+// head + 3 activation maps, at most 32 layers (29 KB of the 32 KB limit).
+constexpr int kMaxStepMaps = 7 * 32 + 4;
+struct StepParams {
+  StepArgs a;
+  CUtensorMap maps[kMaxStepMaps];
+};
+
+// Launch of the persistent kernel (bn_max 32/64/128, head_dim 64/128).
+cudaError_t launch_step_persistent(const StepParams& p, int bn_max, int hd, int grid,
+                                   cudaStream_t s, bool cooperative);
+cudaError_t step_persistent_set_attributes();
+size_t step_persistent_smem_bytes(int bn_max, int hd);
 
 // ---- launchers (kernels.cu) --------------------------------------------------------
 struct GemmMaps {

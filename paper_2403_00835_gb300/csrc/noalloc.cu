@@ -113,6 +113,7 @@ extern "C" int cllm_gemm_bf16_noalloc(const void* W, const void* X, float* Y, in
   g.rows_qk = M;
   g.lo_rows = x_rows;
   g.l2_ahead = 16;
+  g.pre_stages = 1 << 20;
   g.partial = reinterpret_cast<float*>(sb + off_part);
   g.tickets = reinterpret_cast<int*>(sb + off_tick);
   g.err = reinterpret_cast<int*>(sb + off_err);
