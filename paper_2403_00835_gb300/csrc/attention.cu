@@ -113,7 +113,8 @@ __global__ void __launch_bounds__(128) attn_chunk_simt_kernel(const AttnArgs a) 
   }
 }
 
-// Merge of a row's chunk partials 0..pos/128 in chunk order; out = O / l.
+// Merge of a row's chunk partials 0..pos/128 in chunk order; out = O / l
+// (fmaf accumulation in chunk order, as in the persistent kernel's merge).
 template <typename Act>
 __global__ void attn_combine_kernel(const AttnArgs a) {
   pdl_launch_dependents();
@@ -129,8 +130,8 @@ __global__ void attn_combine_kernel(const AttnArgs a) {
     for (int c = 0; c < nch; ++c) {
       const float2 ml = a.part_ml[base + c];
       const float f = exp2f(ml.x - M);
-      l += f * ml.y;
-      acc += f * a.part_o[(base + c) * a.hd + d];
+      l = fmaf(f, ml.y, l);
+      acc = fmaf(f, a.part_o[(base + c) * a.hd + d], acc);
     }
     st_gin(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * a.hd + h * a.hd + d, a.plane_out,
            acc / l);

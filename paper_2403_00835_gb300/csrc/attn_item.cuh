@@ -300,8 +300,13 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
 }
 
 // Merge of the chunk partials 0..pos/128 of every row of query tile qi for
-// head h, in chunk order (the same arithmetic as the attention combine
-// kernel); out = O / l, written as the GEMM input planes.
+// head h, in chunk order; out = O / l, written as the GEMM input planes.
+// Per output element: l = sum_c f_c l_c and acc = sum_c f_c O_c with
+// f_c = 2^(m_c - M), both accumulated with fmaf in chunk order (the attention
+// combine kernel computes the same sums).  Thread (row, part) owns 16 (HD 128)
+// or 8 (HD 64) consecutive dimensions; the partials of 4 chunks are loaded
+// together (the first group with the (m, l) scan), so a row of up to 512 keys
+// costs one round trip.
 template <typename Act, int HD, class Meta>
 __device__ void attn_combine_tile(const AttnArgs& a, int qi, int h, int tid, const Meta& md) {
   const int2 qt = md.qtile(qi);
@@ -309,26 +314,57 @@ __device__ void attn_combine_tile(const AttnArgs& a, int qi, int h, int tid, con
   const int nr = min(kQTile, md.nrows(b) - r0);
   const int row = tid >> 3, part = tid & 7;
   constexpr int DPT = HD / 8;
+  constexpr int NV = DPT / 4;  // float4 per chunk and thread
+  constexpr int CG = 4;        // chunks per load group
   if (row >= nr) return;
   const int t = md.row0(b) + r0 + row;
   const int pos = md.start(b) + r0 + row;  // the row's position (pos[t])
   const int nch = min(pos / kAttnChunk + 1, a.nch_max);
   const size_t base = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
-  float M = -INFINITY;
-  for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&a.part_ml[base + c].x));
+  float2 ml[CG];
+  float4 ov[CG][NV];
+  auto load_group = [&](int c0) {
 #pragma unroll
-  for (int dd = 0; dd < DPT; ++dd) {
-    const int d = part * DPT + dd;
-    float acc = 0.f, l = 0.f;
-    for (int c = 0; c < nch; ++c) {
-      const float2 ml = __ldcg(&a.part_ml[base + c]);
-      const float f = exp2f(ml.x - M);
-      l += f * ml.y;
-      acc += f * __ldcg(&a.part_o[(base + c) * HD + d]);
+    for (int q = 0; q < CG; ++q) {
+      if (c0 + q < nch) {
+        ml[q] = __ldcg(&a.part_ml[base + c0 + q]);
+        const float4* src =
+            reinterpret_cast<const float4*>(a.part_o + (base + c0 + q) * HD + part * DPT);
+#pragma unroll
+        for (int v = 0; v < NV; ++v) ov[q][v] = __ldcg(src + v);
+      }
     }
-    st_gin(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * HD + h * HD + d, a.plane_out,
-           acc / l);
+  };
+  load_group(0);
+  float M = -INFINITY;
+#pragma unroll
+  for (int q = 0; q < CG; ++q)
+    if (q < nch) M = fmaxf(M, ml[q].x);
+  for (int c = CG; c < nch; ++c) M = fmaxf(M, __ldcg(&a.part_ml[base + c].x));
+  float acc[DPT];
+#pragma unroll
+  for (int dd = 0; dd < DPT; ++dd) acc[dd] = 0.f;
+  float l = 0.f;
+  for (int c0 = 0; c0 < nch; c0 += CG) {
+    if (c0 > 0) load_group(c0);
+#pragma unroll
+    for (int q = 0; q < CG; ++q) {
+      if (c0 + q < nch) {
+        const float f = exp2f(ml[q].x - M);
+        l = fmaf(f, ml[q].y, l);
+#pragma unroll
+        for (int v = 0; v < NV; ++v) {
+          acc[4 * v + 0] = fmaf(f, ov[q][v].x, acc[4 * v + 0]);
+          acc[4 * v + 1] = fmaf(f, ov[q][v].y, acc[4 * v + 1]);
+          acc[4 * v + 2] = fmaf(f, ov[q][v].z, acc[4 * v + 2]);
+          acc[4 * v + 3] = fmaf(f, ov[q][v].w, acc[4 * v + 3]);
+        }
+      }
+    }
   }
+  const size_t o = static_cast<size_t>(t) * a.H * HD + h * HD + part * DPT;
+#pragma unroll
+  for (int dd = 0; dd < DPT; ++dd) st_gin(static_cast<Act*>(a.out), o + dd, a.plane_out, acc[dd] / l);
 }
 
 }  // namespace cllm

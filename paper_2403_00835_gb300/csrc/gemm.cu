@@ -43,11 +43,13 @@ namespace cllm {
 template <int BNMAX>
 using SoloCfg = TcCfg<BNMAX, BNMAX <= 32 ? 8 : (BNMAX <= 64 ? 6 : (BNMAX <= 128 ? 4 : 2))>;
 
+constexpr int kSoloRedSlots = 2;  // split-K partial blocks staged per reduction round
+
 template <int BNMAX>
 constexpr size_t solo_smem_bytes() {
   using Cfg = SoloCfg<BNMAX>;
   return 1024 + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES + sizeof(EpiSmem) + 16 +
-         tc_bar_bytes(Cfg::STAGES);
+         kSoloRedSlots * kRedSlotBytes + tc_bar_bytes(Cfg::STAGES);
 }
 
 template <int KIND, int BNMAX>
@@ -60,8 +62,8 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* base =
       reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(base + Cfg::STAGES * Cfg::STAGE_BYTES);
-  uint8_t* bars = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(&es + 1) + 15) & ~uintptr_t(15));
+  float* red = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(&es + 1) + 15) & ~uintptr_t(15));
+  uint8_t* bars = reinterpret_cast<uint8_t*>(red) + kSoloRedSlots * kRedSlotBytes;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&mA0);
@@ -69,7 +71,9 @@ __global__ void __launch_bounds__(192, 1)
     tma_prefetch_desc(&mA2);
     tma_prefetch_desc(&mB);
   }
-  const TcPipe P = tc_pipe_init<Cfg>(base, bars);
+  TcPipe P = tc_pipe_init<Cfg>(base, bars);
+  P.red = red;
+  P.red_slots = kSoloRedSlots;
   // Every CTA of this grid is resident (one per SM): let the next kernel in
   // the stream start its independent prologue now.
   pdl_launch_dependents();

@@ -47,7 +47,13 @@ struct TcPipe {
   uint64_t* drain;
   volatile int* abort;
   uint32_t tmem;
+  // staging of split-K partials for the last arriver's reduction: red_slots
+  // blocks of kEpiCols x kBM floats (set by the kernel after tc_pipe_init)
+  float* red;
+  int red_slots;
 };
+
+constexpr size_t kRedSlotBytes = sizeof(float) * kEpiCols * kBM;
 
 // Shared-memory bytes of the barrier block that follows the ring.
 __host__ __device__ constexpr size_t tc_bar_bytes(int stages) { return 8 * (2 * stages + 5) + 16; }
@@ -419,22 +425,29 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
           float v[kEpiCols];
 #pragma unroll
           for (int j = 0; j < kEpiCols; ++j) v[j] = 0.f;
-          // contributors in slot order; each group's loads are issued together
-          for (int s0 = 0; s0 < nc; s0 += 8) {
-            float w[8][kEpiCols];
+          // Contributors in slot order.  A group of up to red_slots partial
+          // blocks (kEpiCols x kBM contiguous floats each) is copied to shared
+          // memory by all 128 threads at once (cp.async at L2, no registers
+          // held), then each thread adds its row.
+          for (int s0 = 0; s0 < nc; s0 += P.red_slots) {
+            const int ns = min(P.red_slots, nc - s0);
+            for (int q = 0; q < ns; ++q) {
+              const float* src = g.partial + (static_cast<size_t>(u) * g.maxc + s0 + q) * g.bn * kBM +
+                                 static_cast<size_t>(ch) * kEpiCols * kBM;
+              float* dst = P.red + q * (kEpiCols * kBM);
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const float* p = g.partial + (static_cast<size_t>(u) * g.maxc + s0 + q) * g.bn * kBM;
-#pragma unroll
-              for (int j = 0; j < kEpiCols; ++j)
-                w[q][j] = (s0 + q < nc) ? __ldcg(p + (ch * kEpiCols + j) * kBM + r) : 0.f;
+              for (int i = 0; i < kEpiCols * kBM / (4 * 128); ++i)
+                cp_async16(dst + 4 * (i * 128 + r), src + 4 * (i * 128 + r));
             }
+            cp_async_commit();
+            cp_async_wait_all();
+            epi_sync();
+            for (int q = 0; q < ns; ++q) {
+              const float* blk = P.red + q * (kEpiCols * kBM);
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-              if (s0 + q < nc) {
-#pragma unroll
-                for (int j = 0; j < kEpiCols; ++j) v[j] += w[q][j];
-              }
+              for (int j = 0; j < kEpiCols; ++j) v[j] += blk[j * kBM + r];
+            }
+            epi_sync();
           }
           epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
         }

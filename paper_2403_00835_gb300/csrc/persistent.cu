@@ -30,7 +30,12 @@ struct PersistCfg {
   static constexpr size_t ATTN_BYTES = align_up(sizeof(AttnTileSmem<HD>), 16) +
                                        align_up(4 * (kMaxQTilesStep + 1), 16) +
                                        align_up(sizeof(AttnMetaSmem), 16);
-  static constexpr size_t UNION = align_up(ATTN_BYTES > sizeof(EpiSmem) ? ATTN_BYTES : sizeof(EpiSmem), 16);
+  // the GEMM epilogue's part of the union: EpiSmem, then split-K staging
+  // blocks (at least 4; as many as fit beside the attention tile)
+  static constexpr size_t EPI_BYTES = align_up(sizeof(EpiSmem), 16);
+  static constexpr size_t EPI_MIN = EPI_BYTES + 4 * kRedSlotBytes;
+  static constexpr size_t UNION = align_up(ATTN_BYTES > EPI_MIN ? ATTN_BYTES : EPI_MIN, 16);
+  static constexpr int RED_SLOTS = static_cast<int>((UNION - EPI_BYTES) / kRedSlotBytes);
   static constexpr int STAGE_BYTES = kBM * kBK * 2 + 2 * BNMAX * kBK * 2;
   static constexpr size_t BUDGET = 227 * 1024;
   static constexpr size_t FIXED = 1024 + UNION + tc_bar_bytes(8) + 64;
@@ -113,7 +118,9 @@ __global__ void __launch_bounds__(192, 1)
   AttnMetaSmem& meta = *reinterpret_cast<AttnMetaSmem*>(
       uni + align_up(sizeof(AttnTileSmem<HD>), 16) + align_up(4 * (kMaxQTilesStep + 1), 16));
   uint8_t* bars = uni + PC::UNION;
-  const TcPipe P = tc_pipe_init<Cfg>(base, bars);
+  TcPipe P = tc_pipe_init<Cfg>(base, bars);
+  P.red = reinterpret_cast<float*>(uni + PC::EPI_BYTES);
+  P.red_slots = PC::RED_SLOTS;
   const int G = gridDim.x, cta = blockIdx.x;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
