@@ -51,11 +51,22 @@ int cllm_test_gemm_bf16_timed(const void *W, long long w_stride_bytes, int n_w, 
 int cllm_test_phase_stamps(cllm_ctx *ctx, unsigned long long *out, int cap, const char **names,
                            int names_cap);
 
-/* Per-CTA timestamps of the last profiled persistent iteration:
- * out[(k * P + p) * G + cta], k = 0 phase start (dependency seen), 1 MMA
- * issuer done with the phase (GEMM phases), 2 arrival at the grid barrier;
- * G = SM count.  Returns the number of values (3 * P * G). */
+/* Per-CTA timestamps of the last profiled persistent iteration (global
+ * timer, ns): out[(k * P + p) * G + cta] for k = 0..12 -- 0 phase start
+ * (barrier seen), 1 MMA issuer done with the phase (GEMM phases), 2 arrival
+ * at the grid barrier, 3-5 the epilogue's last segment (accumulator ready,
+ * after the split-K ticket, done), 6 producer enters the phase, 8 producer
+ * done, 10/11 first/last stage arrival at the MMA, 12 largest gap between
+ * arrivals (ns); slots 7 and 9 are unused (0).  Then 256 * G traced arrivals
+ * (see cllm_test_set_trace_phase).  G = SM count.  Returns the number of
+ * values, (13 * P + 256) * G. */
 int cllm_test_cta_stamps(cllm_ctx *ctx, unsigned long long *out, long long cap);
+
+/* Profiling: trace every MMA stage arrival (global timer, ns) of phase
+ * `phase` of the persistent kernel, up to 256 per CTA; they follow the
+ * per-CTA stamps in cllm_test_cta_stamps' output ([cta][256], 0 = unused).
+ * -1 turns tracing off.  Drops the captured graphs.  EINVAL on a null ctx. */
+int cllm_test_set_trace_phase(cllm_ctx *ctx, int phase);
 
 #ifdef __cplusplus
 }

@@ -181,6 +181,7 @@ struct cllm_ctx {
   std::vector<unsigned long long> last_stamps;  // last profiled persistent iteration
   std::vector<std::string> last_phase_names;
   std::vector<unsigned long long> last_cta_stamps;
+  int trace_phase = -1;  // profiling: phase whose MMA stage arrivals are traced
   std::map<std::tuple<int, int, int, int, int, unsigned long long, int, int, int, int>, GraphEntry>
       graphs;
   // profiling
@@ -679,7 +680,8 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   void* tk_d = upload(nullptr, static_cast<size_t>(n_qtiles) * c->H * sizeof(int) + 16);
   void* bar_d = upload(nullptr, 64);
   void* st_d = upload(nullptr, (5 * ph.size() + 1) * sizeof(unsigned long long));
-  void* cst_d = upload(nullptr, 6 * ph.size() * c->sms * sizeof(unsigned long long));
+  void* cst_d = upload(nullptr, (kCtaStampSlots * ph.size() + kTraceCap) * c->sms *
+                                    sizeof(unsigned long long));
   if (!ph_d || !tk_d || !bar_d || !st_d || !cst_d) return CLLM_ENOMEM;
   ge.cta_stamps = static_cast<unsigned long long*>(cst_d);
   if (c->profiling) {
@@ -706,6 +708,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   sa.accept = make_accept(c, B, n, mode == MODE_DECODE);
   sa.stamps = c->profiling ? ge.stamps : nullptr;
   sa.cta_stamps = c->profiling ? ge.cta_stamps : nullptr;
+  sa.trace_phase = c->trace_phase;
   sa.err = c->err;
   return CLLM_OK;
 }
@@ -897,7 +900,8 @@ void accumulate_profile(cllm_ctx* c, const cllm_ctx::GraphEntry* ge) {
       return;
     c->last_stamps = st;
     c->last_phase_names = ge->phase_names;
-    c->last_cta_stamps.resize(6 * static_cast<size_t>(ge->n_phases) * c->sms);
+    c->last_cta_stamps.resize((kCtaStampSlots * static_cast<size_t>(ge->n_phases) + kTraceCap) *
+                              c->sms);
     cudaMemcpy(c->last_cta_stamps.data(), ge->cta_stamps, c->last_cta_stamps.size() * 8,
                cudaMemcpyDeviceToHost);
     // phase p runs from CTA 0 seeing its dependency met to the next phase's
@@ -1788,6 +1792,20 @@ extern "C" int cllm_test_phase_stamps(cllm_ctx* c, unsigned long long* out, int 
   for (int i = 0; i < static_cast<int>(c->last_phase_names.size()) && i < names_cap; ++i)
     names[i] = c->last_phase_names[i].c_str();
   return n;
+}
+
+extern "C" int cllm_test_set_trace_phase(cllm_ctx* c, int phase) {
+  if (!c) return CLLM_EINVAL;
+  c->trace_phase = phase;
+  cudaSetDevice(c->dev);
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess) return cuda_fail(cudaGetLastError(), "sync");
+  for (auto& kv : c->graphs) {
+    if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
+    if (kv.second.qtiles) cudaFree(kv.second.qtiles);
+    for (void* p : kv.second.bufs) cudaFree(p);
+  }
+  c->graphs.clear();
+  return CLLM_OK;
 }
 
 extern "C" int cllm_test_cta_stamps(cllm_ctx* c, unsigned long long* out, long long cap) {

@@ -315,8 +315,13 @@ __device__ void tc_produce_drain(const TcPipe& P, int issued) {
 
 template <class Cfg>
 __device__ bool tc_mma(const TcPipe& P, int& idx, int& acc, uint32_t& accph, const GemmArgs& g,
-                       int c0, int c1) {
+                       int c0, int c1, unsigned long long* prof = nullptr, long long prof_stride = 0,
+                       unsigned long long* trace = nullptr) {
   constexpr int S = Cfg::STAGES;
+  // optional profile: first and last stage arrival, largest gap between
+  // arrivals, and (trace) every arrival
+  unsigned long long t_first = 0, t_last = 0, gap = 0;
+  int ntrace = 0;
   const uint32_t idesc = idesc_bf16_f32(kBM, Cfg::STACKED ? 2 * g.bn : g.bn);
   int c = c0;
   Segment sg;
@@ -328,6 +333,13 @@ __device__ bool tc_mma(const TcPipe& P, int& idx, int& acc, uint32_t& accph, con
       const int st = idx % S;
       if (!mbar_wait(&P.full[st], (idx / S) & 1, P.abort)) return false;
       tc_fence_after();
+      if (prof != nullptr) {
+        const unsigned long long now = globaltimer_ns();
+        if (trace != nullptr && ntrace < kTraceCap) trace[ntrace++] = now;
+        if (t_first == 0) t_first = now;
+        else if (now - t_last > gap) gap = now - t_last;
+        t_last = now;
+      }
       const uint32_t a_addr = smem_u32(P.sA + st * Cfg::A_BYTES);
       const uint32_t b_addr = smem_u32(P.sB + st * Cfg::B_BYTES);
 #pragma unroll
@@ -346,6 +358,11 @@ __device__ bool tc_mma(const TcPipe& P, int& idx, int& acc, uint32_t& accph, con
       acc = 0;
       accph ^= 1;
     }
+  }
+  if (prof != nullptr) {
+    prof[0] = t_first;
+    prof[prof_stride] = t_last;
+    prof[2 * prof_stride] = gap;
   }
   return true;
 }

@@ -179,10 +179,17 @@ struct StepArgs {
   int* attn_tickets;        // [qtiles][heads], self-resetting
   AcceptArgs accept;
   unsigned long long* stamps;  // optional: phase start times (CTA 0)
-  unsigned long long* cta_stamps;  // optional: [6][phase][cta] start, MMA done, arrival, epilogue
+  // optional: [kCtaStampSlots][phase][cta] -- epilogue group start, MMA done,
+  // arrival, 3 epilogue stamps, producer start, (unused), producer done,
+  // (unused), first and last stage arrival at the MMA, largest gap between
+  // arrivals (ns); then kTraceCap stage arrivals per CTA of phase trace_phase
+  unsigned long long* cta_stamps;
+  int trace_phase;  // -1: none
   int* err;
 };
 
+constexpr int kCtaStampSlots = 13;
+constexpr int kTraceCap = 256;
 constexpr int kMaxQTilesStep = 256;  // query tiles of one iteration (persistent kernel)
 
 // Tensor maps travel by value in the kernel's parameter space (TMA reads

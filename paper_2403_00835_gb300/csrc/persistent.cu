@@ -90,11 +90,12 @@ __device__ bool epilogue_phase(const TcPipe& P, int& acc, uint32_t& accph, const
 
 template <class Cfg>
 __device__ bool mma_phase(const TcPipe& P, int& idx, int& acc, uint32_t& accph, const PhaseDesc& ph,
-                          int cta) {
+                          int cta, unsigned long long* prof, long long prof_stride,
+                          unsigned long long* trace) {
   const GemmArgs g = ph.g;
   int c0, c1;
   cta_range(g, cta, c0, c1);
-  return tc_mma<Cfg>(P, idx, acc, accph, g, c0, c1);
+  return tc_mma<Cfg>(P, idx, acc, accph, g, c0, c1, prof, prof_stride, trace);
 }
 
 }  // namespace
@@ -132,7 +133,13 @@ __global__ void __launch_bounds__(192, 1)
         const PhaseDesc& ph = A.phases[p];
         if (ph.kind != PH_GEMM) continue;
         const GridDep dep{A.bar, static_cast<unsigned>(p) * static_cast<unsigned>(G)};
-        if (!produce_phase<Cfg>(P, idx, issued, ph, PRM.maps, cta, dep)) break;
+        const size_t PG = static_cast<size_t>(A.n_phases) * G;
+        unsigned long long* cs =
+            A.cta_stamps != nullptr ? A.cta_stamps + static_cast<size_t>(p) * G + cta : nullptr;
+        if (cs != nullptr) cs[6 * PG] = globaltimer_ns();
+        const bool ok = produce_phase<Cfg>(P, idx, issued, ph, PRM.maps, cta, dep);
+        if (cs != nullptr) cs[8 * PG] = globaltimer_ns();
+        if (!ok) break;
       }
       tc_produce_drain<Cfg>(P, issued);
     }
@@ -144,7 +151,15 @@ __global__ void __launch_bounds__(192, 1)
       for (int p = 0; p < A.n_phases; ++p) {
         const PhaseDesc& ph = A.phases[p];
         if (ph.kind != PH_GEMM) continue;
-        if (!mma_phase<Cfg>(P, idx, acc, accph, ph, cta)) break;
+        unsigned long long* prof = nullptr;
+        unsigned long long* trace = nullptr;
+        const long long PG = static_cast<long long>(A.n_phases) * G;
+        if (A.cta_stamps != nullptr) {
+          prof = A.cta_stamps + 10 * PG + static_cast<long long>(p) * G + cta;
+          if (p == A.trace_phase)
+            trace = A.cta_stamps + kCtaStampSlots * PG + static_cast<long long>(cta) * kTraceCap;
+        }
+        if (!mma_phase<Cfg>(P, idx, acc, accph, ph, cta, prof, PG, trace)) break;
         if (A.cta_stamps != nullptr)
           A.cta_stamps[(static_cast<size_t>(A.n_phases) + p) * G + cta] = globaltimer_ns();
       }
