@@ -375,6 +375,35 @@ __device__ __forceinline__ void tc_mma_drain(const TcPipe& P) {
 
 // ---- epilogue (128 threads; r = TMEM lane = weight row of the tile) -------------------
 
+__device__ __forceinline__ void red_release_gpu(int* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Bounded wait until *p >= target (acquire).  On timeout sets *abort.
+__device__ inline bool count_wait(const int* p, int target, volatile int* abort) {
+  const uint64_t t0 = globaltimer_ns();
+  while (static_cast<int>(ld_acquire_gpu(reinterpret_cast<const unsigned*>(p))) < target) {
+    if (*abort) return false;
+    if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+      *abort = 1;
+      return false;
+    }
+    __nanosleep(32);
+  }
+  return true;
+}
+
+
+// hi + lo accumulator columns of 16 token columns (chunk ch) of this thread's row
+template <class Cfg>
+__device__ __forceinline__ void tmem_ld_sum_cfg(uint32_t taddr, int ch, int bn, float (&v)[kEpiCols]) {
+  tmem_ld16(taddr + ch * kEpiCols, v);
+  float vlo[kEpiCols];
+  tmem_ld16(taddr + (Cfg::STACKED ? bn : Cfg::BN) + ch * kEpiCols, vlo);
+#pragma unroll
+  for (int j = 0; j < kEpiCols; ++j) v[j] += vlo[j];
+}
+
 template <int KIND, class Cfg>
 __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const GemmArgs& g,
                             const EpiArgs& e, int c0, int c1, int cta, EpiSmem& es) {
@@ -408,71 +437,79 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     const uint32_t taddr = P.tmem + (static_cast<uint32_t>(grp * 32) << 16) +
                            static_cast<uint32_t>(acc * Cfg::ACC_COLS);
     float* mypart = g.partial + (static_cast<size_t>(u) * g.maxc + slot) * g.bn * kBM;
-    for (int ch = 0; ch < nchunk; ++ch) {
-      float v[kEpiCols];
-      tmem_ld16(taddr + ch * kEpiCols, v);
-      {
-        float vlo[kEpiCols];
-        tmem_ld16(taddr + (Cfg::STACKED ? g.bn : Cfg::BN) + ch * kEpiCols, vlo);
-#pragma unroll
-        for (int j = 0; j < kEpiCols; ++j) v[j] += vlo[j];
-      }
-      if (nc == 1) {
-        epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
-      } else {
-#pragma unroll
-        for (int j = 0; j < kEpiCols; ++j) mypart[(ch * kEpiCols + j) * kBM + r] = v[j];
-      }
-    }
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&P.tempty[acc]);
-    if (nc > 1) {
-      epi_sync();
-      if (r == 0) {
-        const int old = ticket_add(&g.tickets[u], 1);
-        es.flag = (old == nc - 1);
-      }
-      epi_sync();
-      const bool last_arrival = es.flag;
-      epi_sync();
-      if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
-      if (last_arrival) {
-        for (int ch = 0; ch < nchunk; ++ch) {
-          float v[kEpiCols];
-#pragma unroll
-          for (int j = 0; j < kEpiCols; ++j) v[j] = 0.f;
-          // Contributors in slot order.  A group of up to red_slots partial
-          // blocks (kEpiCols x kBM contiguous floats each) is copied to shared
-          // memory by all 128 threads at once (cp.async at L2, no registers
-          // held), then each thread adds its row.
-          for (int s0 = 0; s0 < nc; s0 += P.red_slots) {
-            const int ns = min(P.red_slots, nc - s0);
-            for (int q = 0; q < ns; ++q) {
-              const float* src = g.partial + (static_cast<size_t>(u) * g.maxc + s0 + q) * g.bn * kBM +
-                                 static_cast<size_t>(ch) * kEpiCols * kBM;
-              float* dst = P.red + q * (kEpiCols * kBM);
-#pragma unroll
-              for (int i = 0; i < kEpiCols * kBM / (4 * 128); ++i)
-                cp_async16(dst + 4 * (i * 128 + r), src + 4 * (i * 128 + r));
-            }
-            cp_async_commit();
-            cp_async_wait_all();
-            epi_sync();
-            for (int q = 0; q < ns; ++q) {
-              const float* blk = P.red + q * (kEpiCols * kBM);
-#pragma unroll
-              for (int j = 0; j < kEpiCols; ++j) v[j] += blk[j * kBM + r];
-            }
-            epi_sync();
-          }
+    // Split-K: the unit's contributors are CTAs first..last (slots 0..nc-1).
+    // Slot 0 -- for which this unit is the last segment of its range, so it
+    // finishes with the phase -- owns the reduction: the others store their
+    // partial sums and release a count; the owner waits for nc - 1, then adds
+    // the partials to its own accumulator in slot order.
+    const bool owner = nc > 1 && slot == 0;
+    if (!owner) {
+      for (int ch = 0; ch < nchunk; ++ch) {
+        float v[kEpiCols];
+        tmem_ld_sum_cfg<Cfg>(taddr, ch, g.bn, v);
+        if (nc == 1) {
           epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
+        } else {
+#pragma unroll
+          for (int j = 0; j < kEpiCols; ++j) mypart[(ch * kEpiCols + j) * kBM + r] = v[j];
         }
-        if (r == 0) g.tickets[u] = 0;
-        if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
       }
-    } else if (KIND == EPI_ARGMAX) {
-      epi_argmax_finish(e, r, es);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&P.tempty[acc]);
+      if (nc > 1) {
+        epi_sync();  // every thread's partial stores precede the release
+        if (r == 0) red_release_gpu(&g.tickets[u], 1);
+        if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
+      } else if (KIND == EPI_ARGMAX) {
+        epi_argmax_finish(e, r, es);
+      }
+    } else {
+      if (r == 0) es.ok = count_wait(&g.tickets[u], nc - 1, P.abort) ? 1 : 0;
+      epi_sync();
+      const bool got = es.ok != 0;
+      epi_sync();
+      if (!got) {
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&P.tempty[acc]);
+        return false;
+      }
+      if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
+      for (int ch = 0; ch < nchunk; ++ch) {
+        float v[kEpiCols];
+        tmem_ld_sum_cfg<Cfg>(taddr, ch, g.bn, v);
+        // slots 1..nc-1: a group of up to red_slots partial blocks
+        // (kEpiCols x kBM contiguous floats each) is copied to shared memory
+        // by all 128 threads at once (cp.async at L2, no registers held),
+        // then each thread adds its row
+        for (int s0 = 1; s0 < nc; s0 += P.red_slots) {
+          const int ns = min(P.red_slots, nc - s0);
+          for (int q = 0; q < ns; ++q) {
+            const float* src = g.partial + (static_cast<size_t>(u) * g.maxc + s0 + q) * g.bn * kBM +
+                               static_cast<size_t>(ch) * kEpiCols * kBM;
+            float* dst = P.red + q * (kEpiCols * kBM);
+#pragma unroll
+            for (int i = 0; i < kEpiCols * kBM / (4 * 128); ++i)
+              cp_async16(dst + 4 * (i * 128 + r), src + 4 * (i * 128 + r));
+          }
+          cp_async_commit();
+          cp_async_wait_all();
+          epi_sync();
+          for (int q = 0; q < ns; ++q) {
+            const float* blk = P.red + q * (kEpiCols * kBM);
+#pragma unroll
+            for (int j = 0; j < kEpiCols; ++j) v[j] += blk[j * kBM + r];
+          }
+          epi_sync();
+        }
+        epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&P.tempty[acc]);
+      if (r == 0) g.tickets[u] = 0;
+      if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
     }
     if (dbg) e.dbg[2 * e.dbg_stride + cta] = globaltimer_ns();
     if (++acc == Cfg::NACC) {
