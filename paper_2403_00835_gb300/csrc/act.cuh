@@ -28,6 +28,26 @@ __device__ __forceinline__ void st_gin(__nv_bfloat16* p, size_t i, size_t plane,
   p[i] = hi;
   p[i + plane] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
+// Four consecutive elements (i a multiple of 4): one vector store per plane.
+__device__ __forceinline__ void st_gin4(float* p, size_t i, size_t, float4 v) {
+  *reinterpret_cast<float4*>(p + i) = v;
+}
+__device__ __forceinline__ void st_gin4(__nv_bfloat16* p, size_t i, size_t plane, float4 v) {
+  const float x[4] = {v.x, v.y, v.z, v.w};
+  __nv_bfloat16 hi[4], lo[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    hi[k] = __float2bfloat16_rn(x[k]);
+    lo[k] = __float2bfloat16_rn(x[k] - __bfloat162float(hi[k]));
+  }
+  uint2 h, l;
+  h.x = static_cast<uint32_t>(__bfloat16_as_ushort(hi[0])) | (static_cast<uint32_t>(__bfloat16_as_ushort(hi[1])) << 16);
+  h.y = static_cast<uint32_t>(__bfloat16_as_ushort(hi[2])) | (static_cast<uint32_t>(__bfloat16_as_ushort(hi[3])) << 16);
+  l.x = static_cast<uint32_t>(__bfloat16_as_ushort(lo[0])) | (static_cast<uint32_t>(__bfloat16_as_ushort(lo[1])) << 16);
+  l.y = static_cast<uint32_t>(__bfloat16_as_ushort(lo[2])) | (static_cast<uint32_t>(__bfloat16_as_ushort(lo[3])) << 16);
+  *reinterpret_cast<uint2*>(p + i) = h;
+  *reinterpret_cast<uint2*>(p + i + plane) = l;
+}
 __device__ __forceinline__ float ld_gin(const float* p, size_t i, size_t) { return p[i]; }
 __device__ __forceinline__ float ld_gin(const __nv_bfloat16* p, size_t i, size_t plane) {
   return __bfloat162float(p[i]) + __bfloat162float(p[i + plane]);

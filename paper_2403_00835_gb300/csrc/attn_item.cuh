@@ -260,32 +260,37 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   }
   sync();
   {
-    const int row = tid >> 3, part = tid & 7;
-    constexpr int DPT = HD / 8;
-    if (row < nr) {
-      float M = -INFINITY;
+    // thread -> (row, 4 consecutive dims): a row's HD floats are written by
+    // HD/4 consecutive threads as float4 (coalesced)
+    constexpr int TPR = HD / 4;           // threads per row
+    constexpr int RPP = 128 / TPR;        // rows per pass
+    const int d = (tid % TPR) * 4;
 #pragma unroll
-      for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
-      const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + c;
-      float* dst = a.part_o + pidx * HD + part * DPT;
-      if (M == -INFINITY) {
+    for (int row = tid / TPR; row < kQTile; row += RPP) {
+      if (row < nr) {
+        float M = -INFINITY;
 #pragma unroll
-        for (int dd = 0; dd < DPT; ++dd) dst[dd] = 0.f;
-        if (part == 0) a.part_ml[pidx] = make_float2(-INFINITY, 0.f);
-      } else {
-        float f[4], l = 0.f;
+        for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
+        const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + c;
+        float4* dst = reinterpret_cast<float4*>(a.part_o + pidx * HD + d);
+        if (M == -INFINITY) {
+          *dst = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (d == 0) a.part_ml[pidx] = make_float2(-INFINITY, 0.f);
+        } else {
+          float f[4], l = 0.f;
 #pragma unroll
-        for (int w = 0; w < 4; ++w) {
-          f[w] = exp2f(sm.m[w][row] - M);
-          l += f[w] * sm.l[w][row];
+          for (int w = 0; w < 4; ++w) {
+            f[w] = exp2f(sm.m[w][row] - M);
+            l += f[w] * sm.l[w][row];
+          }
+          float o4[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            o4[k] = ((f[0] * co[0][row][d + k] + f[1] * co[1][row][d + k]) + f[2] * co[2][row][d + k]) +
+                    f[3] * co[3][row][d + k];
+          *dst = make_float4(o4[0], o4[1], o4[2], o4[3]);
+          if (d == 0) a.part_ml[pidx] = make_float2(M, l);
         }
-#pragma unroll
-        for (int dd = 0; dd < DPT; ++dd) {
-          const int d = part * DPT + dd;
-          dst[dd] = ((f[0] * co[0][row][d] + f[1] * co[1][row][d]) + f[2] * co[2][row][d]) +
-                    f[3] * co[3][row][d];
-        }
-        if (part == 0) a.part_ml[pidx] = make_float2(M, l);
       }
     }
   }
@@ -303,68 +308,85 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
 // head h, in chunk order; out = O / l, written as the GEMM input planes.
 // Per output element: l = sum_c f_c l_c and acc = sum_c f_c O_c with
 // f_c = 2^(m_c - M), both accumulated with fmaf in chunk order (the attention
-// combine kernel computes the same sums).  Thread (row, part) owns 16 (HD 128)
-// or 8 (HD 64) consecutive dimensions; the partials of 4 chunks are loaded
-// together (the first group with the (m, l) scan), so a row of up to 512 keys
-// costs one round trip.
+// combine kernel computes the same sums).  Thread -> (row, 4 consecutive
+// dims), HD/4 consecutive threads per row, so loads and stores are coalesced
+// vectors; the rows of all passes and the partials of 2 chunks are loaded
+// together, so a tile of up to 256 keys costs one round trip.
 template <typename Act, int HD, class Meta>
 __device__ void attn_combine_tile(const AttnArgs& a, int qi, int h, int tid, const Meta& md) {
   const int2 qt = md.qtile(qi);
   const int b = qt.x, r0 = qt.y;
   const int nr = min(kQTile, md.nrows(b) - r0);
-  const int row = tid >> 3, part = tid & 7;
-  constexpr int DPT = HD / 8;
-  constexpr int NV = DPT / 4;  // float4 per chunk and thread
-  constexpr int CG = 4;        // chunks per load group
-  if (row >= nr) return;
-  const int t = md.row0(b) + r0 + row;
-  const int pos = md.start(b) + r0 + row;  // the row's position (pos[t])
-  const int nch = min(pos / kAttnChunk + 1, a.nch_max);
-  const size_t base = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
-  float2 ml[CG];
-  float4 ov[CG][NV];
+  constexpr int TPR = HD / 4;        // threads per row
+  constexpr int RPP = 128 / TPR;     // rows per pass
+  constexpr int NP = kQTile / RPP;   // passes
+  constexpr int CG = 2;              // chunks per load group
+  const int d = (tid % TPR) * 4;
+  int nch[NP];
+  size_t base[NP];
+  float2 ml[NP][CG];
+  float4 ov[NP][CG];
   auto load_group = [&](int c0) {
 #pragma unroll
-    for (int q = 0; q < CG; ++q) {
-      if (c0 + q < nch) {
-        ml[q] = __ldcg(&a.part_ml[base + c0 + q]);
-        const float4* src =
-            reinterpret_cast<const float4*>(a.part_o + (base + c0 + q) * HD + part * DPT);
+    for (int ps = 0; ps < NP; ++ps)
 #pragma unroll
-        for (int v = 0; v < NV; ++v) ov[q][v] = __ldcg(src + v);
-      }
-    }
+      for (int q = 0; q < CG; ++q)
+        if (c0 + q < nch[ps]) {
+          ml[ps][q] = __ldcg(&a.part_ml[base[ps] + c0 + q]);
+          ov[ps][q] = __ldcg(reinterpret_cast<const float4*>(a.part_o + (base[ps] + c0 + q) * HD + d));
+        }
   };
+  int nch_max = 0;
+#pragma unroll
+  for (int ps = 0; ps < NP; ++ps) {
+    const int row = ps * RPP + tid / TPR;
+    const int t = md.row0(b) + r0 + row;
+    const int pos = md.start(b) + r0 + row;  // the row's position (pos[t])
+    nch[ps] = row < nr ? min(pos / kAttnChunk + 1, a.nch_max) : 0;
+    base[ps] = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
+    nch_max = max(nch_max, nch[ps]);
+  }
   load_group(0);
-  float M = -INFINITY;
+  float M[NP];
 #pragma unroll
-  for (int q = 0; q < CG; ++q)
-    if (q < nch) M = fmaxf(M, ml[q].x);
-  for (int c = CG; c < nch; ++c) M = fmaxf(M, __ldcg(&a.part_ml[base + c].x));
-  float acc[DPT];
+  for (int ps = 0; ps < NP; ++ps) {
+    M[ps] = -INFINITY;
 #pragma unroll
-  for (int dd = 0; dd < DPT; ++dd) acc[dd] = 0.f;
-  float l = 0.f;
-  for (int c0 = 0; c0 < nch; c0 += CG) {
+    for (int q = 0; q < CG; ++q)
+      if (q < nch[ps]) M[ps] = fmaxf(M[ps], ml[ps][q].x);
+    for (int c = CG; c < nch[ps]; ++c) M[ps] = fmaxf(M[ps], __ldcg(&a.part_ml[base[ps] + c].x));
+  }
+  float4 acc[NP];
+  float l[NP];
+#pragma unroll
+  for (int ps = 0; ps < NP; ++ps) {
+    acc[ps] = make_float4(0.f, 0.f, 0.f, 0.f);
+    l[ps] = 0.f;
+  }
+  for (int c0 = 0; c0 < nch_max; c0 += CG) {
     if (c0 > 0) load_group(c0);
 #pragma unroll
-    for (int q = 0; q < CG; ++q) {
-      if (c0 + q < nch) {
-        const float f = exp2f(ml[q].x - M);
-        l = fmaf(f, ml[q].y, l);
+    for (int ps = 0; ps < NP; ++ps)
 #pragma unroll
-        for (int v = 0; v < NV; ++v) {
-          acc[4 * v + 0] = fmaf(f, ov[q][v].x, acc[4 * v + 0]);
-          acc[4 * v + 1] = fmaf(f, ov[q][v].y, acc[4 * v + 1]);
-          acc[4 * v + 2] = fmaf(f, ov[q][v].z, acc[4 * v + 2]);
-          acc[4 * v + 3] = fmaf(f, ov[q][v].w, acc[4 * v + 3]);
+      for (int q = 0; q < CG; ++q)
+        if (c0 + q < nch[ps]) {
+          const float f = exp2f(ml[ps][q].x - M[ps]);
+          l[ps] = fmaf(f, ml[ps][q].y, l[ps]);
+          acc[ps].x = fmaf(f, ov[ps][q].x, acc[ps].x);
+          acc[ps].y = fmaf(f, ov[ps][q].y, acc[ps].y);
+          acc[ps].z = fmaf(f, ov[ps][q].z, acc[ps].z);
+          acc[ps].w = fmaf(f, ov[ps][q].w, acc[ps].w);
         }
-      }
-    }
   }
-  const size_t o = static_cast<size_t>(t) * a.H * HD + h * HD + part * DPT;
 #pragma unroll
-  for (int dd = 0; dd < DPT; ++dd) st_gin(static_cast<Act*>(a.out), o + dd, a.plane_out, acc[dd] / l);
+  for (int ps = 0; ps < NP; ++ps) {
+    const int row = ps * RPP + tid / TPR;
+    if (row >= nr) continue;
+    const int t = md.row0(b) + r0 + row;
+    const float L = l[ps];
+    st_gin4(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * HD + h * HD + d, a.plane_out,
+            make_float4(acc[ps].x / L, acc[ps].y / L, acc[ps].z / L, acc[ps].w / L));
+  }
 }
 
 }  // namespace cllm
