@@ -17,8 +17,10 @@ decode (n = 1) is timed the same way.  ``--impl reference`` times the oracle
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -109,6 +111,36 @@ def dist_setup():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return world, rank, local
+
+
+def kernel_sources_digest():
+    """First 16 hex digits of the SHA-256 of the CUDA sources (names and contents)."""
+    h = hashlib.sha256()
+    src = os.path.join(ROOT, "paper_2403_00835_gb300", "csrc")
+    for name in sorted(os.listdir(src)):
+        if name.endswith((".cu", ".cuh")):
+            h.update(name.encode())
+            with open(os.path.join(src, name), "rb") as f:
+                h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def measured_traffic(kernel, workload, layers):
+    """DRAM bytes (read + write) per launch of `kernel` from the committed ncu
+    summary of this workload, or None when there is none or the kernel sources
+    changed since it was taken."""
+    if layers:
+        return None
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload.replace('-', '_')}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    m = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    d = re.search(r"kernel_sources_sha256_16:\s*([0-9a-f]{16})", text)
+    if not m or not d or d.group(1) != kernel_sources_digest():
+        return None
+    return float(m.group(1))
 
 
 def step_bytes(cfg, B, n, L_mean):
@@ -289,6 +321,12 @@ def run_ours(args, world, rank, local):
     out, iters = eng.jacobi_decode(prompts, n, max_new, seed=2)
     e2e_s = time.perf_counter() - t0
     e2e_val = float(np.sum(out >= 0)) * world / e2e_s
+    e2e_iters = max(1, int(np.max(iters)))
+    # host<->device bytes of that call, per decode iteration: the prompt
+    # tokens and lengths in, the status word (12 bytes) out every iteration,
+    # and the committed tokens and iteration counts out at the end
+    e2e_h2d = 4 * (sum(lens) + B) / e2e_iters
+    e2e_d2h = 12 + 4 * (B * max_new + B) / e2e_iters
 
     hbm, tflops, peak_kind = measured_peaks()
     T = B * n
@@ -319,15 +357,17 @@ def run_ours(args, world, rank, local):
                               "peak_gbs": hbm, "frac": sbytes / (ms_step / 1e3) / 1e9 / hbm,
                               "peak_kind": peak_kind},
         "roofline": {"bound": "hbm", "kernel": k_name, "achieved": achieved, "peak": hbm,
-                     "unit": "GB/s", "frac": (achieved / hbm) if achieved else None, "traffic": None,
+                     "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
+                     "traffic": measured_traffic(k_name, args.workload, args.layers),
                      "peak_kind": f"{peak_kind} (copy bandwidth)",
                      "algorithmic_bytes_per_launch": k_bytes, "avg_launch_ms": k_avg},
         "kernel_share": {k: round(v[0] / tot_prof, 4) for k, v in sorted(phases.items())} if tot_prof else {},
         "kernel_avg_us": {k: round(1e3 * v[0] / max(v[1], 1), 2) for k, v in sorted(phases.items())},
         "persistent_kernel": persistent,
         "e2e": {"value": e2e_val, "unit": "tokens/s",
-                "h2d_bytes_per_step": 4 * (sum(lens) + B), "d2h_bytes_per_step": 4 * (B * max_new + B),
-                "what": f"cllm_jacobi_decode of {B}x{max_new} tokens incl. prefill, wall clock"},
+                "h2d_bytes_per_step": e2e_h2d, "d2h_bytes_per_step": e2e_d2h,
+                "what": f"cllm_jacobi_decode of {B}x{max_new} tokens incl. prefill, wall clock, "
+                        f"host buffers; {e2e_iters} iterations"},
         "gpu_launches": launches_per_iter * args.steps + rs_j,
         "clocks": clocks,
     }
