@@ -52,6 +52,8 @@ extern "C" {
 #define CLLM_GUESS_UNIFORM 0      /* initial/refill guesses uniform over the vocab   */
 #define CLLM_GUESS_FROM_PROMPT 1  /* guesses drawn from the prompt's tokens (Alg. 3) */
 #define CLLM_BLOCK_REFILL 0       /* block stays n wide: fresh guesses after commits */
+#define CLLM_BLOCK_SHRINK 1       /* Alg. 3: the window narrows by the accepted tokens
+                                     until it is fixed, then a fresh n-wide block */
 
 /*
  * Model shape and capacity.  The decoder is the pre-norm LLaMA layer:
@@ -91,7 +93,9 @@ typedef struct {
   uint64_t seed;   /* key of the counter-based guess generator                    */
   int eos_id;      /* -1: off.  Else a sequence stops after committing this token   */
   int guess_init;  /* CLLM_GUESS_UNIFORM | CLLM_GUESS_FROM_PROMPT                  */
-  int block_mode;  /* CLLM_BLOCK_REFILL (the only policy of this build)            */
+  int block_mode;  /* CLLM_BLOCK_REFILL | CLLM_BLOCK_SHRINK                       */
+  int record_cap;  /* > 0: record the first record_cap blocks of every sequence
+                      (the Jacobi trajectory), read with cllm_decode_read_trajectory */
 } cllm_decode_opts;
 
 typedef struct cllm_ctx cllm_ctx;
@@ -197,6 +201,14 @@ int cllm_decode_run(cllm_ctx *ctx, int max_iters, int *iters_run, int64_t *commi
 /* Copy out the decode's tokens [B][max_new] (-1 past the end) and the
  * per-sequence iteration counts [B] (either may be NULL). */
 int cllm_decode_read(cllm_ctx *ctx, int32_t *tokens_out, int32_t *iters_out);
+
+/* Copy out the recorded trajectory (Sec. 3.1: the sequence of blocks
+ * y^(0), y^(1), ... of Jacobi decoding; Alg. 3 with the decode's block
+ * policy): blocks_out[it][b][k] for it < record_cap of cllm_decode_begin's
+ * options, k < n; slots beyond a shrunken window and iterations a sequence
+ * did not run are -1.  Host buffer of record_cap*B*n ints, owned by the
+ * caller.  ESTATE when the decode did not record. */
+int cllm_decode_read_trajectory(cllm_ctx *ctx, int32_t *blocks_out);
 
 /* ---- options --------------------------------------------------------------------
  * CLLM_OPT_PERSISTENT (default 1): run each decode/step iteration of the bf16

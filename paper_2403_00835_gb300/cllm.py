@@ -21,13 +21,15 @@ STATUS = {0: "CLLM_OK", -1: "CLLM_EINVAL", -2: "CLLM_ENOMEM", -3: "CLLM_ECUDA", 
 CLLM_F32, CLLM_BF16 = 0, 1
 CLLM_GUESS_UNIFORM, CLLM_GUESS_FROM_PROMPT = 0, 1
 CLLM_BLOCK_REFILL = 0
+CLLM_BLOCK_SHRINK = 1
 
 # Every function declared in include/cllm.h.
 EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode",
            "cllm_ar_decode", "cllm_status_string", "cllm_decode_begin", "cllm_decode_run",
            "cllm_decode_read", "cllm_set_profiling", "cllm_profile_read",
            "cllm_kernels_per_iteration", "cllm_committed_lengths", "cllm_gemm_bf16_noalloc",
-           "cllm_set_option", "cllm_uses_persistent", "cllm_last_cuda_error")
+           "cllm_set_option", "cllm_uses_persistent", "cllm_last_cuda_error",
+           "cllm_decode_read_trajectory")
 CLLM_OPT_PERSISTENT = 1
 CLLM_OPT_L2_AHEAD = 2
 CLLM_OPT_PRE_STAGES = 3
@@ -59,7 +61,7 @@ class Weights(ctypes.Structure):
 
 class DecodeOpts(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("eos_id", ctypes.c_int), ("guess_init", ctypes.c_int),
-                ("block_mode", ctypes.c_int)]
+                ("block_mode", ctypes.c_int), ("record_cap", ctypes.c_int)]
 
 
 _lib = None
@@ -110,6 +112,7 @@ def load(build_if_missing: bool = True):
     lib.cllm_set_option.restype = ctypes.c_int
     lib.cllm_uses_persistent.argtypes = [vp, ctypes.c_int]
     lib.cllm_uses_persistent.restype = ctypes.c_int
+    lib.cllm_decode_read_trajectory.argtypes = [vp, i32p]
     lib.cllm_last_cuda_error.argtypes = []
     lib.cllm_last_cuda_error.restype = ctypes.c_char_p
     for name in ("cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode", "cllm_ar_decode",
@@ -225,15 +228,23 @@ class Engine:
         return {"next": nxt, "accepted": acc, "gap": gap, "logits": lg}
 
     def jacobi_decode(self, prompts, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
-                      guess_init: int = CLLM_GUESS_UNIFORM):
+                      guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL,
+                      record_cap: int = 0):
+        """Tokens [B][max_new] and iterations [B]; with record_cap > 0 also the
+        trajectory [record_cap][B][n] (-1 outside the window)."""
         toks, lens = _flatten_prompts(prompts)
         B = len(prompts)
         out = np.zeros((B, max_new), dtype=np.int32)
         its = np.zeros(B, dtype=np.int32)
-        o = DecodeOpts(seed, eos_id, guess_init, CLLM_BLOCK_REFILL)
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, record_cap)
         _check(self._lib.cllm_jacobi_decode(self._h, B, _ip(toks), _ip(lens), n, max_new,
                                             ctypes.byref(o), _ip(out), _ip(its)), "cllm_jacobi_decode")
         self.B = B
+        if record_cap > 0:
+            traj = np.zeros((record_cap, B, n), dtype=np.int32)
+            _check(self._lib.cllm_decode_read_trajectory(self._h, _ip(traj)),
+                   "cllm_decode_read_trajectory")
+            return out, its, traj
         return out, its
 
     def ar_decode(self, prompts, max_new: int, eos_id: int = -1):
@@ -246,8 +257,8 @@ class Engine:
         return out
 
     def decode_begin(self, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
-                     guess_init: int = CLLM_GUESS_UNIFORM):
-        o = DecodeOpts(seed, eos_id, guess_init, CLLM_BLOCK_REFILL)
+                     guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL):
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, 0)
         _check(self._lib.cllm_decode_begin(self._h, n, max_new, ctypes.byref(o)), "cllm_decode_begin")
         self._dec_max_new = max_new
 

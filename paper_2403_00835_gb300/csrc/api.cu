@@ -151,8 +151,11 @@ struct cllm_ctx {
   // sequence state
   int *Ld = nullptr, *head = nullptr, *head0 = nullptr, *block = nullptr, *committed = nullptr,
       *iters = nullptr, *done = nullptr, *out = nullptr, *accepted = nullptr, *prompts = nullptr,
-      *plen = nullptr, *status = nullptr, *err = nullptr;
+      *plen = nullptr, *status = nullptr, *err = nullptr, *width = nullptr;
   size_t out_cap = 0;
+  int* traj = nullptr;  // recorded trajectory [traj_cap][B][n]
+  size_t traj_alloc = 0;
+  int traj_cap = 0;
   int* status_host = nullptr;  // pinned: slots of 4 ints {active, committed, device error, -}
   cudaEvent_t iter_ev[2] = {nullptr, nullptr};
   // host state
@@ -513,6 +516,10 @@ AcceptArgs make_accept(cllm_ctx* c, int B, int n, bool decode) {
   a.plen = c->plen;
   a.prompt_ld = c->arch.max_seq;
   a.status = c->status;
+  a.shrink = (decode && c->dec_opts.block_mode == CLLM_BLOCK_SHRINK) ? 1 : 0;
+  a.width = c->width;
+  a.traj = (decode && c->traj_cap > 0) ? c->traj : nullptr;
+  a.traj_cap = decode ? c->traj_cap : 0;
   return a;
 }
 
@@ -724,7 +731,10 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
   auto key = std::make_tuple(mode, B, n, mode == MODE_DECODE ? c->dec_max_new : 0,
                              mode == MODE_DECODE ? c->dec_opts.eos_id : 0,
                              mode == MODE_DECODE ? static_cast<unsigned long long>(c->dec_opts.seed) : 0ull,
-                             mode == MODE_DECODE ? c->dec_opts.guess_init : 0, c->profiling ? 1 : 0,
+                             mode == MODE_DECODE ? (c->dec_opts.guess_init | (c->dec_opts.block_mode << 2) |
+                                                    (c->traj_cap << 4))
+                                                 : 0,
+                             c->profiling ? 1 : 0,
                              c->persistent ? 1 : 0, c->l2_ahead_persistent * 65536 + std::min(c->pre_stages, 65535));
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
@@ -1150,6 +1160,7 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
          dev_alloc(c, &c->head0, Bm * 4) && dev_alloc(c, &c->block, Bm * a.max_block * 4) &&
          dev_alloc(c, &c->committed, Bm * 4) && dev_alloc(c, &c->iters, Bm * 4) &&
          dev_alloc(c, &c->done, Bm * 4) && dev_alloc(c, &c->accepted, Bm * 4) &&
+         dev_alloc(c, &c->width, Bm * 4) &&
          dev_alloc(c, &c->prompts, Bm * a.max_seq * 4) && dev_alloc(c, &c->plen, Bm * 4) &&
          dev_alloc(c, &c->status, 16) && dev_alloc(c, &c->err, 16);
     if (!ok) {
@@ -1370,17 +1381,30 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
   o.block_mode = CLLM_BLOCK_REFILL;
   if (opts) o = *opts;
   if (o.guess_init != CLLM_GUESS_UNIFORM && o.guess_init != CLLM_GUESS_FROM_PROMPT) return CLLM_EINVAL;
-  if (o.block_mode != CLLM_BLOCK_REFILL) return CLLM_EUNSUPPORTED;
+  if (o.block_mode != CLLM_BLOCK_REFILL && o.block_mode != CLLM_BLOCK_SHRINK) return CLLM_EINVAL;
+  if (o.record_cap < 0 || o.record_cap > (1 << 20)) return CLLM_EINVAL;
   if (o.eos_id >= c->V) return CLLM_EINVAL;
   for (int b = 0; b < c->B; ++b)
     if (static_cast<long>(c->lens[b]) + max_new + n > c->arch.max_seq) return CLLM_ECAPACITY;
   cudaSetDevice(c->dev);
   const size_t need = static_cast<size_t>(c->B) * max_new;
+  const size_t traj_need = static_cast<size_t>(o.record_cap) * c->B * n;
+  bool stale = false;
+  if (traj_need > c->traj_alloc) {
+    int* p = nullptr;
+    if (!dev_alloc(c, &p, traj_need * 4)) return CLLM_ENOMEM;
+    c->traj = p;
+    c->traj_alloc = traj_need;
+    stale = true;
+  }
   if (need > c->out_cap) {
     int* p = nullptr;
     if (!dev_alloc(c, &p, need * 4)) return CLLM_ENOMEM;
     c->out = p;
     c->out_cap = need;
+    stale = true;
+  }
+  if (stale) {
     // graphs captured against the old output buffer are stale
     for (auto& kv : c->graphs) {
       if (kv.second.exec) cudaGraphExecDestroy(kv.second.exec);
@@ -1392,6 +1416,9 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
   c->dec_n = n;
   c->dec_max_new = max_new;
   c->dec_opts = o;
+  c->traj_cap = o.record_cap;
+  if (traj_need > 0 && cudaMemsetAsync(c->traj, 0xff, traj_need * 4, c->stream) != cudaSuccess)
+    return CLLM_ECUDA;
   if (cudaMemcpyAsync(c->head, c->head0, c->B * 4, cudaMemcpyDeviceToDevice, c->stream) !=
       cudaSuccess)
     return CLLM_ECUDA;
@@ -1477,6 +1504,16 @@ extern "C" int cllm_decode_read(cllm_ctx* c, int32_t* tokens_out, int32_t* iters
   if (iters_out &&
       cudaMemcpyAsync(iters_out, c->iters, c->B * 4, cudaMemcpyDeviceToHost, c->stream))
     return CLLM_ECUDA;
+  return check_device_error(c);
+}
+
+extern "C" int cllm_decode_read_trajectory(cllm_ctx* c, int32_t* blocks_out) {
+  if (!c || !blocks_out) return CLLM_EINVAL;
+  if (!c->dec_active || c->traj_cap <= 0) return CLLM_ESTATE;
+  cudaSetDevice(c->dev);
+  const size_t bytes = static_cast<size_t>(c->traj_cap) * c->B * c->dec_n * 4;
+  if (cudaMemcpyAsync(blocks_out, c->traj, bytes, cudaMemcpyDeviceToHost, c->stream) != cudaSuccess)
+    return cuda_fail(cudaGetLastError(), "trajectory copy");
   return check_device_error(c);
 }
 

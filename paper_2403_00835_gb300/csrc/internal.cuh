@@ -153,6 +153,14 @@ struct AcceptArgs {
   const int* plen;
   int prompt_ld;
   int* status;  // [0] active sequences, [1] tokens committed by this iteration
+  // block policy (Alg. 3): 0 refill (always n wide), 1 shrink (the window
+  // narrows by the accepted count until it is fixed, then a fresh n-wide block)
+  int shrink;
+  int* width;  // [B] current block width (shrink)
+  // optional trajectory: traj[it][b][k] = the block of sequence b at its
+  // iteration it (slot k < width, -1 beyond), for it < traj_cap
+  int* traj;
+  int traj_cap;
 };
 
 // ---- persistent per-iteration kernel (persistent.cu) ---------------------------------

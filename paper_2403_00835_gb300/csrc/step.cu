@@ -41,6 +41,7 @@ __global__ void __launch_bounds__(128) decode_init_kernel(const AcceptArgs a) {
     a.committed[b] = 0;
     a.iters[b] = 0;
     a.done[b] = 0;
+    if (a.width != nullptr) a.width[b] = a.n;
     int* y = a.block + b * a.n;
     y[0] = a.head[b];
     for (int k = 1; k < a.n; ++k) y[k] = draw_guess(a, b, 0, k);

@@ -79,8 +79,13 @@ __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, 
     const int* P = a.pred + b * n;
     int* y = a.block + b * n;
     if (!(a.decode && a.done[b])) {
+      const int w = (a.decode && a.shrink) ? a.width[b] : n;  // active rows of the block
+      if (a.decode && a.traj != nullptr && a.iters[b] < a.traj_cap) {
+        int* tr = a.traj + (static_cast<size_t>(a.iters[b]) * a.B + b) * n;
+        for (int k = 0; k < n; ++k) tr[k] = k < w ? y[k] : -1;
+      }
       int acc = 1;
-      while (acc < n && y[acc] == P[acc - 1]) ++acc;
+      while (acc < w && y[acc] == P[acc - 1]) ++acc;
       if (a.decode) {
         bool stop = false;
         if (a.eos >= 0) {
@@ -104,11 +109,23 @@ __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, 
       a.accepted[b] = acc;
       a.L[b] += acc;
       a.head[b] = P[acc - 1];
-      if (a.decode) {
+      if (a.decode && !a.shrink) {
         // next block: the predictions from the new head on, then fresh guesses
         const int keep = n - acc + 1;
         const int step = a.iters[b];
         for (int k = 0; k < n; ++k) y[k] = (k < keep) ? P[acc - 1 + k] : draw_guess(a, b, step, k);
+      } else if (a.decode) {
+        const int step = a.iters[b];
+        if (acc == w) {
+          // the whole window is fixed: a fresh block, the new head then guesses
+          for (int k = 0; k < n; ++k) y[k] = (k == 0) ? P[acc - 1] : draw_guess(a, b, step, k);
+          a.width[b] = n;
+        } else {
+          // the window narrows to the positions not yet fixed; rows beyond it
+          // are computed but ignored (they hold valid tokens)
+          for (int k = 0; k < n; ++k) y[k] = P[min(acc - 1 + k, n - 1)];
+          a.width[b] = w - acc;
+        }
       }
     }
   }
