@@ -115,6 +115,27 @@ __device__ __forceinline__ int ticket_add(int* p, int v) {
   return old;
 }
 
+// Column sums of a warp: every lane holds one value per column (16 columns);
+// the result for column c = lane >> 1 ends in lanes 2c and 2c + 1.  Halving
+// exchanges (16 shuffles in 5 independent rounds) instead of 16 separate
+// 5-shuffle trees; the association order is fixed.
+__device__ __forceinline__ float warp_colsum16(const float (&v)[kEpiCols], int lane) {
+  static_assert(kEpiCols == 16, "16 columns");
+  float a[8], b[4], c[2];
+  const bool h16 = lane & 16, h8 = lane & 8, h4 = lane & 4, h2 = lane & 2;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    a[i] = (h16 ? v[i + 8] : v[i]) + __shfl_xor_sync(0xffffffffu, h16 ? v[i] : v[i + 8], 16);
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    b[i] = (h8 ? a[i + 4] : a[i]) + __shfl_xor_sync(0xffffffffu, h8 ? a[i] : a[i + 4], 8);
+#pragma unroll
+  for (int i = 0; i < 2; ++i)
+    c[i] = (h4 ? b[i + 2] : b[i]) + __shfl_xor_sync(0xffffffffu, h4 ? b[i] : b[i + 2], 4);
+  float d = (h2 ? c[1] : c[0]) + __shfl_xor_sync(0xffffffffu, h2 ? c[0] : c[1], 2);
+  return d + __shfl_xor_sync(0xffffffffu, d, 1);
+}
+
 // (max, argmax with lowest index on ties, second max) merge
 __device__ __forceinline__ void am_merge(float& v1, int& i1, float& v2, float w1, int j1, float w2) {
   const bool other_hi = (w1 > v1) || (w1 == v1 && j1 < i1);
@@ -257,10 +278,11 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
   } else if (KIND == EPI_RESID) {
     const int m = mt * kBM + r;
     const float gn = use_pre ? pre->g : ld_act(reinterpret_cast<const Act*>(e.gnext), m);
+    float sq[kEpiCols];
 #pragma unroll
     for (int j = 0; j < kEpiCols; ++j) {
       const int t = t0 + j;
-      float sq = 0.f;
+      sq[j] = 0.f;
       if (t < e.T) {
         const size_t o = static_cast<size_t>(t) * e.d + m;
         // L2 read: other CTAs rewrite the residual stream in earlier phases
@@ -268,11 +290,11 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
         const float xi = (use_pre ? pre->a[j] : __ldcg(e.x + o)) + v[j];
         e.x[o] = xi;
         st_gin(reinterpret_cast<Act*>(e.xg), o, e.plane_x, xi * gn);
-        sq = xi * xi;
+        sq[j] = xi * xi;
       }
-      sq = warp_sum(sq);
-      if (lane == 0) s.red[grp][j] = sq;
     }
+    const float col = warp_colsum16(sq, lane);
+    if ((lane & 1) == 0) s.red[grp][lane >> 1] = col;
     epi_sync();
     if (r < kEpiCols) {
       const int t = t0 + r;
@@ -285,24 +307,47 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
     epi_norm_scale(e, t0, r, s);
     const int m = mt * kBM + r;
     const bool vrow = m < e.V;
+    // per column (max, argmax, second max) over the warp's 32 rows, by the
+    // same halving exchanges as warp_colsum16 (the merge is exact, so the
+    // order does not matter); column c ends in lanes 2c, 2c + 1
+    float c1[kEpiCols], c2[kEpiCols];
+    int ci[kEpiCols];
 #pragma unroll
     for (int j = 0; j < kEpiCols; ++j) {
       const int t = t0 + j;
       const float lg = v[j] * s.rs[j];
       if (e.logits != nullptr && t < e.T && vrow) e.logits[static_cast<size_t>(t) * e.V + m] = lg;
-      float v1 = vrow ? lg : -INFINITY, v2 = -INFINITY;
-      int i1 = m;
+      c1[j] = vrow ? lg : -INFINITY;
+      c2[j] = -INFINITY;
+      ci[j] = m;
+    }
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float w1 = __shfl_xor_sync(0xffffffffu, v1, o);
-        const int j1 = __shfl_xor_sync(0xffffffffu, i1, o);
-        const float w2 = __shfl_xor_sync(0xffffffffu, v2, o);
-        am_merge(v1, i1, v2, w1, j1, w2);
+    for (int o = 16, half = 8; o >= 2; o >>= 1, half >>= 1) {
+      const bool hi = lane & o;
+#pragma unroll
+      for (int i = 0; i < half; ++i) {
+        // keep column i (low lanes) or i + half (high lanes), merge the
+        // partner's copy of it (selects between statically indexed values)
+        const float w1 = __shfl_xor_sync(0xffffffffu, hi ? c1[i] : c1[i + half], o);
+        const int wj = __shfl_xor_sync(0xffffffffu, hi ? ci[i] : ci[i + half], o);
+        const float w2 = __shfl_xor_sync(0xffffffffu, hi ? c2[i] : c2[i + half], o);
+        float a1 = hi ? c1[i + half] : c1[i], a2 = hi ? c2[i + half] : c2[i];
+        int ai = hi ? ci[i + half] : ci[i];
+        am_merge(a1, ai, a2, w1, wj, w2);
+        c1[i] = a1;
+        ci[i] = ai;
+        c2[i] = a2;
       }
-      if (lane == 0) {
-        s.am[grp][j][0] = v1;
-        s.am[grp][j][1] = __int_as_float(i1);
-        s.am[grp][j][2] = v2;
+    }
+    {
+      float a1 = c1[0], a2 = c2[0];
+      int ai = ci[0];
+      am_merge(a1, ai, a2, __shfl_xor_sync(0xffffffffu, c1[0], 1),
+               __shfl_xor_sync(0xffffffffu, ci[0], 1), __shfl_xor_sync(0xffffffffu, c2[0], 1));
+      if ((lane & 1) == 0) {
+        s.am[grp][lane >> 1][0] = a1;
+        s.am[grp][lane >> 1][1] = __int_as_float(ai);
+        s.am[grp][lane >> 1][2] = a2;
       }
     }
     epi_sync();

@@ -494,6 +494,9 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
               cp_async16(dst + 4 * (i * 128 + r), src + 4 * (i * 128 + r));
           }
           cp_async_commit();
+          // the chunk's own epilogue inputs travel in the same round trip
+          if (ch > 0 && s0 == 1)
+            epi_prefetch<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, r, es, pre);
           cp_async_wait_all();
           epi_sync();
           for (int q = 0; q < ns; ++q) {
