@@ -157,3 +157,30 @@ def test_errors_are_reported(pair):
     with pytest.raises(CllmError) as e:
         eng.jacobi_step([[0] * 17])  # n > max_block
     assert e.value.status == -1
+
+
+@pytest.mark.parametrize("n", [32, 48, 64])
+def test_wide_block_step(n):
+    """Blocks of 2-4 query tiles per sequence: the tensor-core attention runs a
+    group of tiles against each staged key chunk; logits and tokens against the
+    oracle, batch 2 with ragged prompts."""
+    cfg = syn.TINY_BF16
+    w_cpu = syn.make_weights(cfg, seed=0, device="cpu")
+    eng = engine_for(cfg, syn.weights_to(w_cpu, "cuda"), max_batch=2, max_seq=256, max_block=64)
+    om = oracle_for(cfg, w_cpu)
+    try:
+        prompts = syn.make_prompts(cfg.vocab, [150, 37], seed=11)
+        guesses = syn.make_guesses(cfg.vocab, len(prompts), n, seed=12)
+        eng.prefill(prompts)
+        r = eng.jacobi_step(guesses, want_gap=True, want_logits=True)
+        for b, p in enumerate(prompts):
+            s = om.session(256)
+            head, _, _ = orc.prefill(s, p)
+            st = orc.jacobi_step(s, [head] + guesses[b][1:], len(p), keep_logits=True)
+            ok, worst = logits_ok(r["logits"][b], st.logits, cfg.dtype)
+            assert ok, f"b={b} logits err/bound={worst:.3g}"
+            for k in range(n):
+                if st.gap[k] >= FLAG_GAP:
+                    assert r["next"][b][k] == st.pred[k], (b, k)
+    finally:
+        eng.close()
