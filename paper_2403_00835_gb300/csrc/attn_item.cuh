@@ -13,7 +13,7 @@ namespace cllm {
 template <int HD>
 struct AttnTileSmem {
   __half q[kQTile][HD + 8];
-  __half k[kAttnChunk][HD + 8];  // reused as float co[4][kQTile][HD] for the warp merge
+  __half k[kAttnChunk][HD + 8];  // reused as float co[4][kQTile][HD + 8] for the warp merge
   __half v[kAttnChunk][HD + 8];
   float m[4][kQTile];
   float l[4][kQTile];
@@ -113,7 +113,10 @@ __device__ __forceinline__ int attn_find_qtile(const int* pre, int n, int item) 
 template <int HD, class Sync, class Meta = GlobalMeta>
 __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
                               int tid, Sync sync, int& qi_out, int& h_out, const Meta& md) {
-  static_assert(sizeof(float) * 4 * kQTile * HD <= sizeof(__half) * kAttnChunk * (HD + 8),
+  // merge area: rows padded by 8 floats, so that the 8 row groups of a warp's
+  // accumulator fragment fall in distinct banks
+  constexpr int CLD = HD + 8;
+  static_assert(sizeof(float) * 4 * kQTile * CLD <= sizeof(__half) * kAttnChunk * (HD + 8),
                 "merge area must fit in the K tile");
   const int warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, cq = lane & 3;
@@ -122,7 +125,7 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   const __half* Q = static_cast<const __half*>(a.q);
   const __half* KC = static_cast<const __half*>(a.k_cache);
   const __half* VC = static_cast<const __half*>(a.v_cache);
-  float (*co)[kQTile][HD] = reinterpret_cast<float (*)[kQTile][HD]>(&sm.k[0][0]);
+  float (*co)[kQTile][CLD] = reinterpret_cast<float (*)[kQTile][CLD]>(&sm.k[0][0]);
   const int qi = attn_find_qtile(pre, a.n_qtiles, item);
   const int local = item - pre[qi];
   const int c = local / a.H, h = local - c * a.H;
@@ -247,10 +250,8 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
 #pragma unroll
   for (int dn = 0; dn < HD / 8; ++dn) {
     const int d0 = dn * 8 + 2 * cq;
-    co[warp][g][d0] = o[dn][0];
-    co[warp][g][d0 + 1] = o[dn][1];
-    co[warp][g + 8][d0] = o[dn][2];
-    co[warp][g + 8][d0 + 1] = o[dn][3];
+    *reinterpret_cast<float2*>(&co[warp][g][d0]) = make_float2(o[dn][0], o[dn][1]);
+    *reinterpret_cast<float2*>(&co[warp][g + 8][d0]) = make_float2(o[dn][2], o[dn][3]);
   }
   if (cq == 0) {
     sm.m[warp][g] = mA;
@@ -283,12 +284,14 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
             f[w] = exp2f(sm.m[w][row] - M);
             l += f[w] * sm.l[w][row];
           }
-          float o4[4];
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            o4[k] = ((f[0] * co[0][row][d + k] + f[1] * co[1][row][d + k]) + f[2] * co[2][row][d + k]) +
-                    f[3] * co[3][row][d + k];
-          *dst = make_float4(o4[0], o4[1], o4[2], o4[3]);
+          const float4 w0 = *reinterpret_cast<const float4*>(&co[0][row][d]);
+          const float4 w1 = *reinterpret_cast<const float4*>(&co[1][row][d]);
+          const float4 w2 = *reinterpret_cast<const float4*>(&co[2][row][d]);
+          const float4 w3 = *reinterpret_cast<const float4*>(&co[3][row][d]);
+          *dst = make_float4(((f[0] * w0.x + f[1] * w1.x) + f[2] * w2.x) + f[3] * w3.x,
+                             ((f[0] * w0.y + f[1] * w1.y) + f[2] * w2.y) + f[3] * w3.y,
+                             ((f[0] * w0.z + f[1] * w1.z) + f[2] * w2.z) + f[3] * w3.z,
+                             ((f[0] * w0.w + f[1] * w1.w) + f[2] * w2.w) + f[3] * w3.w);
           if (d == 0) a.part_ml[pidx] = make_float2(M, l);
         }
       }

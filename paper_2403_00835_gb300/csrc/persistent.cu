@@ -27,23 +27,25 @@ __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + 
 
 template <int BNMAX, int HD>
 struct PersistCfg {
-  static constexpr size_t ATTN_BYTES = align_up(sizeof(AttnTileSmem<HD>), 16) +
-                                       align_up(4 * (kMaxQTilesStep + 1), 16) +
-                                       align_up(sizeof(AttnMetaSmem), 16);
+  static constexpr size_t ATTN_BYTES = align_up(sizeof(AttnTileSmem<HD>), 16);
   // the GEMM epilogue's part of the union: EpiSmem, then split-K staging
   // blocks (at least 4; as many as fit beside the attention tile)
   static constexpr size_t EPI_BYTES = align_up(sizeof(EpiSmem), 16);
   static constexpr size_t EPI_MIN = EPI_BYTES + 4 * kRedSlotBytes;
   static constexpr size_t UNION = align_up(ATTN_BYTES > EPI_MIN ? ATTN_BYTES : EPI_MIN, 16);
   static constexpr int RED_SLOTS = static_cast<int>((UNION - EPI_BYTES) / kRedSlotBytes);
+  // the attention work-item prefix and the iteration's metadata, outside the
+  // union: computed at the first attention phase, kept for every layer
+  static constexpr size_t PRE_BYTES = align_up(4 * (kMaxQTilesStep + 1), 16);
+  static constexpr size_t META_BYTES = PRE_BYTES + align_up(sizeof(AttnMetaSmem), 16);
   static constexpr int STAGE_BYTES = kBM * kBK * 2 + 2 * BNMAX * kBK * 2;
   static constexpr size_t BUDGET = 227 * 1024;
-  static constexpr size_t FIXED = 1024 + UNION + tc_bar_bytes(8) + 64;
+  static constexpr size_t FIXED = 1024 + UNION + META_BYTES + tc_bar_bytes(8) + 64;
   static constexpr int FIT = static_cast<int>((BUDGET - FIXED) / STAGE_BYTES);
   static constexpr int STAGES = FIT > 8 ? 8 : FIT;
   using Cfg = TcCfg<BNMAX, STAGES>;
-  static constexpr size_t SMEM =
-      1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + UNION + tc_bar_bytes(STAGES) + 64;
+  static constexpr size_t SMEM = 1024 + static_cast<size_t>(STAGES) * STAGE_BYTES + UNION +
+                                 META_BYTES + tc_bar_bytes(STAGES) + 64;
   static_assert(STAGES >= 2, "ring too small");
   static_assert(SMEM <= BUDGET, "shared memory over budget");
 };
@@ -115,10 +117,9 @@ __global__ void __launch_bounds__(192, 1)
   uint8_t* uni = base + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES;
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(uni);
   AttnTileSmem<HD>& at = *reinterpret_cast<AttnTileSmem<HD>*>(uni);
-  int* pre = reinterpret_cast<int*>(uni + align_up(sizeof(AttnTileSmem<HD>), 16));
-  AttnMetaSmem& meta = *reinterpret_cast<AttnMetaSmem*>(
-      uni + align_up(sizeof(AttnTileSmem<HD>), 16) + align_up(4 * (kMaxQTilesStep + 1), 16));
-  uint8_t* bars = uni + PC::UNION;
+  int* pre = reinterpret_cast<int*>(uni + PC::UNION);
+  AttnMetaSmem& meta = *reinterpret_cast<AttnMetaSmem*>(uni + PC::UNION + PC::PRE_BYTES);
+  uint8_t* bars = uni + PC::UNION + PC::META_BYTES;
   TcPipe P = tc_pipe_init<Cfg>(base, bars);
   P.red = reinterpret_cast<float*>(uni + PC::EPI_BYTES);
   P.red_slots = PC::RED_SLOTS;
@@ -171,6 +172,7 @@ __global__ void __launch_bounds__(192, 1)
     const EpiGroupSync sync;
     int acc = 0;
     uint32_t accph = 0;
+    int attn_total = -1;  // attention work items of this iteration (prefix in smem)
     for (int p = 0; p < A.n_phases; ++p) {
       const PhaseDesc& ph = A.phases[p];
       const int kind = ph.kind;
@@ -205,10 +207,13 @@ __global__ void __launch_bounds__(192, 1)
         AttnArgs a = A.attn;
         a.k_cache = ph.k_cache;
         a.v_cache = ph.v_cache;
-        attn_meta_load(a, meta, r, A.accept.B);
-        sync();
         const SmemMeta md{meta};
-        const int total = attn_item_prefix(a, pre, r, sync, md);
+        if (attn_total < 0) {  // the first attention phase of the launch
+          attn_meta_load(a, meta, r, A.accept.B);
+          sync();
+          attn_total = attn_item_prefix(a, pre, r, sync, md);
+        }
+        const int total = attn_total;
         for (int item = cta; item < total; item += G) {
           int qi, h;
           attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md);
