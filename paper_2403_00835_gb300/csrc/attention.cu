@@ -19,6 +19,8 @@
 // in warp order.  fp32: a SIMT kernel with a per-row online softmax.
 #include <float.h>
 
+#include <type_traits>
+
 #include "act.cuh"
 #include "attn_item.cuh"
 #include "internal.cuh"
@@ -47,7 +49,7 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
   const int total = attn_item_prefix(a, sm.pre, threadIdx.x, CtaSync{});
   for (int item = blockIdx.x; item < total; item += gridDim.x) {
     int qi, h;
-    attn_mma_item<HD>(a, item, sm.pre, sm.t, threadIdx.x, CtaSync{}, qi, h);
+    attn_mma_item<HD>(a, item, sm.pre, sm.t, threadIdx.x, CtaSync{}, qi, h, false);
   }
 }
 
@@ -58,7 +60,7 @@ __global__ void __launch_bounds__(128) attn_chunk_simt_kernel(const AttnArgs a) 
   pdl_launch_dependents();
   pdl_wait();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int total = attn_item_prefix(a, pre, threadIdx.x, CtaSync{});
+  const int total = attn_item_prefix(a, pre, threadIdx.x, CtaSync{}, 1);
   const int group = a.H / a.Hkv;
   const int ldq = a.H * HD;
   constexpr int DPL = HD / 32;
@@ -113,15 +115,18 @@ __global__ void __launch_bounds__(128) attn_chunk_simt_kernel(const AttnArgs a) 
   }
 }
 
-// Merge of a row's chunk partials 0..pos/128 in chunk order; out = O / l
+// Merge of a row's partials (per chunk range) in order; out = O / l
 // (fmaf accumulation in chunk order, as in the persistent kernel's merge).
 template <typename Act>
 __global__ void attn_combine_kernel(const AttnArgs a) {
   pdl_launch_dependents();
   pdl_wait();
+  // the tensor-core path leaves one partial per range of kAttnRange chunks,
+  // the fp32 path one per chunk
+  constexpr int R = std::is_same<Act, float>::value ? 1 : kAttnRange;
   const int t = blockIdx.x / a.H, h = blockIdx.x - (blockIdx.x / a.H) * a.H;
   if (t >= a.T) return;
-  const int nch = min(a.pos[t] / kAttnChunk + 1, a.nch_max);
+  const int nch = (min(a.pos[t] / kAttnChunk + 1, a.nch_max) + R - 1) / R;
   const size_t base = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
   float M = -INFINITY;
   for (int c = 0; c < nch; ++c) M = fmaxf(M, a.part_ml[base + c].x);

@@ -71,14 +71,16 @@ __device__ __forceinline__ int attn_tile_chunks(const AttnArgs& a, int qi) {
 }
 
 // Prefix sum of work items over query tiles into pre[0..n_qtiles];
-// items(q) = H * chunks(q).  Warp 0 of the group scans; returns the total.
+// items(q) = H * ceil(chunks(q) / range), range = chunks per item (1 for the
+// per-chunk fp32 path).  Warp 0 of the group scans; returns the total.
 template <class Sync, class Meta = GlobalMeta>
-__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync, const Meta& md) {
+__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync, const Meta& md,
+                                int range = kAttnRange) {
   if (tid < 32) {
     int carry = 0;
     for (int base = 0; base < a.n_qtiles; base += 32) {
       const int q = base + tid;
-      const int cnt = q < a.n_qtiles ? a.H * attn_tile_chunks(a, md, q) : 0;
+      const int cnt = q < a.n_qtiles ? a.H * ((attn_tile_chunks(a, md, q) + range - 1) / range) : 0;
       int incl = cnt;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
@@ -94,8 +96,9 @@ __device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync,
   return pre[a.n_qtiles];
 }
 template <class Sync>
-__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync) {
-  return attn_item_prefix(a, pre, tid, sync, GlobalMeta{a});
+__device__ int attn_item_prefix(const AttnArgs& a, int* pre, int tid, Sync sync,
+                                int range = kAttnRange) {
+  return attn_item_prefix(a, pre, tid, sync, GlobalMeta{a}, range);
 }
 
 __device__ __forceinline__ int attn_find_qtile(const int* pre, int n, int item) {
@@ -108,11 +111,25 @@ __device__ __forceinline__ int attn_find_qtile(const int* pre, int n, int item) 
   return lo;
 }
 
-// Work item `item`: writes the unnormalised chunk partial (O, m, l) of the
-// tile's rows for one head.  Returns the tile index and head in qi_out, h_out.
+// Rows of query tile qi and their number of chunk ranges (the last row's).
+template <class Meta>
+__device__ __forceinline__ int attn_tile_ranges(const AttnArgs& a, const Meta& md, int qi) {
+  return (attn_tile_chunks(a, md, qi) + kAttnRange - 1) / kAttnRange;
+}
+
+// Work item `item`: one (query tile, head, range of kAttnRange key chunks).
+// The 4 warps split each 128-key chunk (32 keys each) and keep an online
+// softmax over the range's chunks; K of the next chunk is loaded while the
+// current chunk's P.V runs, V while the next Q.K runs.  Then the warps' (m, l,
+// O) are merged.  A tile with a single range writes its attention output
+// (O / l, the GEMM input planes) directly and returns true when direct_ok;
+// otherwise the range's partial (O, m, l) goes to slot `range` of the
+// partials (merged by the combine, which gives the same bits for one range).
+// Returns the tile index and head in qi_out, h_out.
 template <int HD, class Sync, class Meta = GlobalMeta>
-__device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
-                              int tid, Sync sync, int& qi_out, int& h_out, const Meta& md) {
+__device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
+                              int tid, Sync sync, int& qi_out, int& h_out, const Meta& md,
+                              bool direct_ok = true) {
   // merge area: rows padded by 8 floats, so that the 8 row groups of a warp's
   // accumulator fragment fall in distinct banks
   constexpr int CLD = HD + 8;
@@ -128,24 +145,35 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   float (*co)[kQTile][CLD] = reinterpret_cast<float (*)[kQTile][CLD]>(&sm.k[0][0]);
   const int qi = attn_find_qtile(pre, a.n_qtiles, item);
   const int local = item - pre[qi];
-  const int c = local / a.H, h = local - c * a.H;
+  const int rg = local / a.H, h = local - rg * a.H;
+  const int nrange = attn_tile_ranges(a, md, qi);
   const int2 qt = md.qtile(qi);
   const int b = qt.x, r0 = qt.y;
   const int nr = min(kQTile, md.nrows(b) - r0);
   const int start = md.start(b);
   const int row_g0 = md.row0(b) + r0;
   const int pos0 = start + r0;  // position of tile row 0
-  const int kb = c * kAttnChunk;
-  int ke = min(kb + kAttnChunk, pos0 + nr);
-  if (ke > a.max_seq) {
-    if (tid == 0) atomicOr(a.err, DERR_CAPACITY);
-    ke = a.max_seq;
-  }
+  const int c0 = rg * kAttnRange;
+  const int c1 = min(c0 + kAttnRange, attn_tile_chunks(a, md, qi));
+  const int kend = min(pos0 + nr, a.max_seq);  // keys of the tile: [0, kend)
+  if (pos0 + nr > a.max_seq && tid == 0) atomicOr(a.err, DERR_CAPACITY);
   const int kvh = h / group;
   const size_t kvbase = ((static_cast<size_t>(b) * a.Hkv + kvh) * a.max_seq) * HD;
-
-  // ---- stage Q (16 rows), K and V (chunk rows) into shared memory ----
   constexpr int CPR = HD * 2 / 16;  // 16-byte pieces per row
+
+  auto load_kv = [&](__half (*dstm)[HD + 8], const __half* src, int c) {
+    const int kb = c * kAttnChunk;
+    for (int i = tid; i < kAttnChunk * CPR; i += 128) {
+      const int rr = i / CPR, pc = i - rr * CPR;
+      void* dst = &dstm[rr][pc * 8];
+      if (kb + rr < kend)
+        cp_async16(dst, src + kvbase + static_cast<size_t>(kb + rr) * HD + pc * 8);
+      else
+        *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+    }
+  };
+
+  // ---- Q (16 rows) and the first chunk's K: group 1; its V: group 2 ----
   for (int i = tid; i < kQTile * CPR; i += 128) {
     const int rr = i / CPR, pc = i - rr * CPR;
     void* dst = &sm.q[rr][pc * 8];
@@ -154,99 +182,120 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
     else
       *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
   }
-  for (int i = tid; i < kAttnChunk * CPR; i += 128) {
-    const int rr = i / CPR, pc = i - rr * CPR;
-    const int key = kb + rr;
-    void* dk = &sm.k[rr][pc * 8];
-    void* dv = &sm.v[rr][pc * 8];
-    if (key < ke) {
-      const size_t off = kvbase + static_cast<size_t>(key) * HD + pc * 8;
-      cp_async16(dk, KC + off);
-      cp_async16(dv, VC + off);
-    } else {
-      *reinterpret_cast<uint4*>(dk) = make_uint4(0, 0, 0, 0);
-      *reinterpret_cast<uint4*>(dv) = make_uint4(0, 0, 0, 0);
-    }
-  }
+  load_kv(sm.k, KC, c0);
   cp_async_commit();
-  cp_async_wait_all();
-  sync();
+  load_kv(sm.v, VC, c0);
+  cp_async_commit();
 
-  // ---- per warp: 32 keys x 16 rows ----
-  const int wk0 = warp * 32;  // first key of this warp, relative to kb
+  const int wk0 = warp * 32;  // first key of this warp within a chunk
+  const int posA = pos0 + g, posB = pos0 + g + 8;
+  const bool rowA = g < nr, rowB = g + 8 < nr;
   float o[HD / 8][4];
 #pragma unroll
   for (int dn = 0; dn < HD / 8; ++dn) o[dn][0] = o[dn][1] = o[dn][2] = o[dn][3] = 0.f;
   float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
-  if (kb + wk0 < ke) {
-    float s[4][4];
+  for (int c = c0; c < c1; ++c) {
+    const int kb = c * kAttnChunk;
+    cp_async_wait_but1();  // Q and this chunk's K
+    sync();
+    float sc[4][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.f;
+    for (int j = 0; j < 4; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
+    const bool live = kb + wk0 < kend;
+    if (live) {
 #pragma unroll
-    for (int ks = 0; ks < HD / 16; ks += 2) {
-      uint32_t qa0[4], qa1[4];
-      ldmatrix_x4(qa0, &sm.q[lane & 15][ks * 16 + (lane >> 4) * 8]);
-      ldmatrix_x4(qa1, &sm.q[lane & 15][(ks + 1) * 16 + (lane >> 4) * 8]);
+      for (int ks = 0; ks < HD / 16; ks += 2) {
+        uint32_t qa0[4], qa1[4];
+        ldmatrix_x4(qa0, &sm.q[lane & 15][ks * 16 + (lane >> 4) * 8]);
+        ldmatrix_x4(qa1, &sm.q[lane & 15][(ks + 1) * 16 + (lane >> 4) * 8]);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          uint32_t kb4[4];
+          const int mi = lane >> 3;
+          ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
+          mma_f16_16816(sc[j], qa0, kb4[0], kb4[1]);
+          mma_f16_16816(sc[j], qa1, kb4[2], kb4[3]);
+        }
+      }
+    }
+    sync();  // every warp is done with K
+    if (c + 1 < c1) load_kv(sm.k, KC, c + 1);
+    cp_async_commit();  // (possibly empty) group: the next chunk's K
+    if (live) {
+      // mask + scale (log2 domain), online softmax over the range's chunks
+      float nA = mA, nB = mB;
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        uint32_t kb4[4];
-        const int mi = lane >> 3;
-        ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
-        mma_f16_16816(s[j], qa0, kb4[0], kb4[1]);
-        mma_f16_16816(s[j], qa1, kb4[2], kb4[3]);
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int key = kb + wk0 + 8 * j + 2 * cq + (e & 1);
+          const bool top = e < 2;
+          const bool valid = key < kend && (top ? (rowA && key <= posA) : (rowB && key <= posB));
+          sc[j][e] = valid ? sc[j][e] * a.scale_log2 : -INFINITY;
+        }
+        nA = fmaxf(nA, fmaxf(sc[j][0], sc[j][1]));
+        nB = fmaxf(nB, fmaxf(sc[j][2], sc[j][3]));
       }
-    }
-    // mask + scale (log2 domain)
-    const int posA = pos0 + g, posB = pos0 + g + 8;
-    const bool rowA = g < nr, rowB = g + 8 < nr;
+      nA = fmaxf(nA, __shfl_xor_sync(0xffffffffu, nA, 1));
+      nA = fmaxf(nA, __shfl_xor_sync(0xffffffffu, nA, 2));
+      nB = fmaxf(nB, __shfl_xor_sync(0xffffffffu, nB, 1));
+      nB = fmaxf(nB, __shfl_xor_sync(0xffffffffu, nB, 2));
+      const float uA = (nA == -INFINITY) ? 0.f : nA;
+      const float uB = (nB == -INFINITY) ? 0.f : nB;
+      const float fA = exp2f(mA - uA), fB = exp2f(mB - uB);  // rescale of the running sums
+      mA = nA;
+      mB = nB;
+      float sA = 0.f, sB = 0.f;
+      uint32_t pa[2][4];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = kb + wk0 + 8 * j + 2 * cq + (e & 1);
-        const bool top = e < 2;
-        const bool valid = key < ke && (top ? (rowA && key <= posA) : (rowB && key <= posB));
-        s[j][e] = valid ? s[j][e] * a.scale_log2 : -INFINITY;
+      for (int j = 0; j < 4; ++j) {
+        const float p0 = exp2f(sc[j][0] - uA), p1 = exp2f(sc[j][1] - uA);
+        const float p2 = exp2f(sc[j][2] - uB), p3 = exp2f(sc[j][3] - uB);
+        sA += p0 + p1;
+        sB += p2 + p3;
+        pa[j >> 1][(j & 1) * 2 + 0] = pack_f16x2(p0, p1);
+        pa[j >> 1][(j & 1) * 2 + 1] = pack_f16x2(p2, p3);
       }
-      mA = fmaxf(mA, fmaxf(s[j][0], s[j][1]));
-      mB = fmaxf(mB, fmaxf(s[j][2], s[j][3]));
-    }
-    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 1));
-    mA = fmaxf(mA, __shfl_xor_sync(0xffffffffu, mA, 2));
-    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 1));
-    mB = fmaxf(mB, __shfl_xor_sync(0xffffffffu, mB, 2));
-    const float uA = (mA == -INFINITY) ? 0.f : mA;
-    const float uB = (mB == -INFINITY) ? 0.f : mB;
-    uint32_t pa[2][4];
+      sA += __shfl_xor_sync(0xffffffffu, sA, 1);
+      sA += __shfl_xor_sync(0xffffffffu, sA, 2);
+      sB += __shfl_xor_sync(0xffffffffu, sB, 1);
+      sB += __shfl_xor_sync(0xffffffffu, sB, 2);
+      lA = lA * fA + sA;
+      lB = lB * fB + sB;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float p0 = exp2f(s[j][0] - uA), p1 = exp2f(s[j][1] - uA);
-      const float p2 = exp2f(s[j][2] - uB), p3 = exp2f(s[j][3] - uB);
-      lA += p0 + p1;
-      lB += p2 + p3;
-      pa[j >> 1][(j & 1) * 2 + 0] = pack_f16x2(p0, p1);
-      pa[j >> 1][(j & 1) * 2 + 1] = pack_f16x2(p2, p3);
-    }
-    lA += __shfl_xor_sync(0xffffffffu, lA, 1);
-    lA += __shfl_xor_sync(0xffffffffu, lA, 2);
-    lB += __shfl_xor_sync(0xffffffffu, lB, 1);
-    lB += __shfl_xor_sync(0xffffffffu, lB, 2);
-    // O = P V: A fragments of P for keys 16kk..16kk+15 are the S accumulators
-    // of n-tiles 2kk, 2kk+1 (a0: row g keys 2c.., a1: row g+8, a2/a3: +8 keys).
-#pragma unroll
-    for (int kk = 0; kk < 2; ++kk) {
-      const uint32_t af[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
-#pragma unroll
-      for (int dn = 0; dn < HD / 8; dn += 2) {
-        uint32_t vb[4];
-        const int mi = lane >> 3;
-        ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
-        mma_f16_16816(o[dn], af, vb[0], vb[1]);
-        mma_f16_16816(o[dn + 1], af, vb[2], vb[3]);
+      for (int dn = 0; dn < HD / 8; ++dn) {
+        o[dn][0] *= fA;
+        o[dn][1] *= fA;
+        o[dn][2] *= fB;
+        o[dn][3] *= fB;
       }
+      cp_async_wait_but1();  // this chunk's V (the next K may be in flight)
+      sync();
+      // O += P V: A fragments of P for keys 16kk..16kk+15 are the S
+      // accumulators of n-tiles 2kk, 2kk+1 (a0: row g keys 2c.., a1: row g+8,
+      // a2/a3: +8 keys).
+#pragma unroll
+      for (int kk = 0; kk < 2; ++kk) {
+        const uint32_t af[4] = {pa[kk][0], pa[kk][1], pa[kk][2], pa[kk][3]};
+#pragma unroll
+        for (int dn = 0; dn < HD / 8; dn += 2) {
+          uint32_t vb[4];
+          const int mi = lane >> 3;
+          ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
+          mma_f16_16816(o[dn], af, vb[0], vb[1]);
+          mma_f16_16816(o[dn + 1], af, vb[2], vb[3]);
+        }
+      }
+    } else {
+      cp_async_wait_but1();
+      sync();
     }
+    sync();  // every warp is done with V
+    if (c + 1 < c1) load_kv(sm.v, VC, c + 1);
+    cp_async_commit();  // (possibly empty) group: the next chunk's V
   }
-  sync();  // every warp is done reading K/V before the merge area overwrites K
+  cp_async_wait_all();
+  sync();
 #pragma unroll
   for (int dn = 0; dn < HD / 8; ++dn) {
     const int d0 = dn * 8 + 2 * cq;
@@ -260,11 +309,12 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
     sm.l[warp][g + 8] = lB;
   }
   sync();
+  const bool single = direct_ok && nrange == 1;
   {
     // thread -> (row, 4 consecutive dims): a row's HD floats are written by
     // HD/4 consecutive threads as float4 (coalesced)
-    constexpr int TPR = HD / 4;           // threads per row
-    constexpr int RPP = 128 / TPR;        // rows per pass
+    constexpr int TPR = HD / 4;     // threads per row
+    constexpr int RPP = 128 / TPR;  // rows per pass
     const int d = (tid % TPR) * 4;
 #pragma unroll
     for (int row = tid / TPR; row < kQTile; row += RPP) {
@@ -272,13 +322,11 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
         float M = -INFINITY;
 #pragma unroll
         for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
-        const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + c;
-        float4* dst = reinterpret_cast<float4*>(a.part_o + pidx * HD + d);
-        if (M == -INFINITY) {
-          *dst = make_float4(0.f, 0.f, 0.f, 0.f);
-          if (d == 0) a.part_ml[pidx] = make_float2(-INFINITY, 0.f);
-        } else {
-          float f[4], l = 0.f;
+        const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + rg;
+        float4 ov = make_float4(0.f, 0.f, 0.f, 0.f);
+        float l = 0.f;
+        if (M != -INFINITY) {
+          float f[4];
 #pragma unroll
           for (int w = 0; w < 4; ++w) {
             f[w] = exp2f(sm.m[w][row] - M);
@@ -288,10 +336,18 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
           const float4 w1 = *reinterpret_cast<const float4*>(&co[1][row][d]);
           const float4 w2 = *reinterpret_cast<const float4*>(&co[2][row][d]);
           const float4 w3 = *reinterpret_cast<const float4*>(&co[3][row][d]);
-          *dst = make_float4(((f[0] * w0.x + f[1] * w1.x) + f[2] * w2.x) + f[3] * w3.x,
-                             ((f[0] * w0.y + f[1] * w1.y) + f[2] * w2.y) + f[3] * w3.y,
-                             ((f[0] * w0.z + f[1] * w1.z) + f[2] * w2.z) + f[3] * w3.z,
-                             ((f[0] * w0.w + f[1] * w1.w) + f[2] * w2.w) + f[3] * w3.w);
+          ov = make_float4(((f[0] * w0.x + f[1] * w1.x) + f[2] * w2.x) + f[3] * w3.x,
+                           ((f[0] * w0.y + f[1] * w1.y) + f[2] * w2.y) + f[3] * w3.y,
+                           ((f[0] * w0.z + f[1] * w1.z) + f[2] * w2.z) + f[3] * w3.z,
+                           ((f[0] * w0.w + f[1] * w1.w) + f[2] * w2.w) + f[3] * w3.w);
+        }
+        if (single) {
+          // the tile's only range: the attention output itself
+          st_gin4(static_cast<__nv_bfloat16*>(a.out),
+                  static_cast<size_t>(row_g0 + row) * a.H * HD + h * HD + d, a.plane_out,
+                  make_float4(ov.x / l, ov.y / l, ov.z / l, ov.w / l));
+        } else {
+          *reinterpret_cast<float4*>(a.part_o + pidx * HD + d) = ov;
           if (d == 0) a.part_ml[pidx] = make_float2(M, l);
         }
       }
@@ -300,15 +356,17 @@ __device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   sync();
   qi_out = qi;
   h_out = h;
+  return single;
 }
 template <int HD, class Sync>
-__device__ void attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
-                              int tid, Sync sync, int& qi_out, int& h_out) {
-  attn_mma_item<HD>(a, item, pre, sm, tid, sync, qi_out, h_out, GlobalMeta{a});
+__device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
+                              int tid, Sync sync, int& qi_out, int& h_out, bool direct_ok) {
+  return attn_mma_item<HD>(a, item, pre, sm, tid, sync, qi_out, h_out, GlobalMeta{a}, direct_ok);
 }
 
-// Merge of the chunk partials 0..pos/128 of every row of query tile qi for
-// head h, in chunk order; out = O / l, written as the GEMM input planes.
+// Merge of the range partials 0..ceil((pos/128 + 1) / kAttnRange) - 1 of every
+// row of query tile qi for head h, in range order; out = O / l, written as the
+// GEMM input planes.
 // Per output element: l = sum_c f_c l_c and acc = sum_c f_c O_c with
 // f_c = 2^(m_c - M), both accumulated with fmaf in chunk order (the attention
 // combine kernel computes the same sums).  Thread -> (row, 4 consecutive
@@ -345,7 +403,7 @@ __device__ void attn_combine_tile(const AttnArgs& a, int qi, int h, int tid, con
     const int row = ps * RPP + tid / TPR;
     const int t = md.row0(b) + r0 + row;
     const int pos = md.start(b) + r0 + row;  // the row's position (pos[t])
-    nch[ps] = row < nr ? min(pos / kAttnChunk + 1, a.nch_max) : 0;
+    nch[ps] = row < nr ? (min(pos / kAttnChunk + 1, a.nch_max) + kAttnRange - 1) / kAttnRange : 0;
     base[ps] = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
     nch_max = max(nch_max, nch[ps]);
   }

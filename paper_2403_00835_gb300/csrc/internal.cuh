@@ -16,6 +16,10 @@ enum : int {
 };
 
 constexpr int kAttnChunk = 128;  // keys per attention chunk, anchored at absolute positions
+// Tensor-core attention: a work item covers a range of kAttnRange consecutive
+// chunks (anchored the same way, so a row's split does not depend on the
+// block size); partials are per range.
+constexpr int kAttnRange = 4;
 constexpr int kQTile = 16;       // query rows per attention tile
 constexpr int kBK = 64;          // K elements per pipeline stage (128 B of bf16)
 constexpr int kBM = 128;         // weight rows per tile (MMA M)

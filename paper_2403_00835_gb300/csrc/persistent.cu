@@ -216,12 +216,12 @@ __global__ void __launch_bounds__(192, 1)
         const int total = attn_total;
         for (int item = cta; item < total; item += G) {
           int qi, h;
-          attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md);
-          // the last chunk of (tile, head) to finish merges the tile's chunks
+          if (attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md)) continue;  // output written
+          // the last range of (tile, head) to finish merges the tile's ranges
           sync();
           if (r == 0) {
             const int old = ticket_add(&A.attn_tickets[qi * a.H + h], 1);
-            s_flag = (old == attn_tile_chunks(a, md, qi) - 1) ? 1 : 0;
+            s_flag = (old == attn_tile_ranges(a, md, qi) - 1) ? 1 : 0;
           }
           sync();
           const bool last = s_flag != 0;
