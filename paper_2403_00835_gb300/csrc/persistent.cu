@@ -237,9 +237,9 @@ __global__ void __launch_bounds__(192, 1)
       if (!ok) break;
       if (p + 1 < A.n_phases) {
         // this CTA's global writes of phase p are read next by other CTAs,
-        // some through TMA (async proxy)
+        // some through TMA (async proxy); thread 0's release after the
+        // barrier covers every thread's writes
         asm volatile("fence.proxy.async.global;" ::: "memory");
-        __threadfence();
         sync();
         if (r == 0) {
           if (A.stamps != nullptr) {
@@ -250,7 +250,7 @@ __global__ void __launch_bounds__(192, 1)
             if (A.cta_stamps != nullptr)
               A.cta_stamps[(2 * static_cast<size_t>(A.n_phases) + p) * G + cta] = now;
           }
-          atomicAdd(A.bar, 1u);
+          asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(A.bar) : "memory");
         }
       }
     }
