@@ -68,6 +68,29 @@ int cllm_test_cta_stamps(cllm_ctx *ctx, unsigned long long *out, long long cap);
  * -1 turns tracing off.  Drops the captured graphs.  EINVAL on a null ctx. */
 int cllm_test_set_trace_phase(cllm_ctx *ctx, int phase);
 
+/*
+ * Failure injection for the bounded on-device waits.  From the next captured
+ * iteration on, the grid barrier of the persistent kernel before phase
+ * `phase` (1 <= phase < the iteration's phase count; phase 0 has no barrier)
+ * waits for one arrival more than the grid makes.  Every CTA's wait there
+ * runs out after the kernel's wait budget (2 s), the CTA waits for its own
+ * copies and tensor-core operations in flight, frees its tensor memory and
+ * returns, and the call that ran the iteration returns CLLM_ETIMEOUT.  No
+ * phase from `phase` on runs, so the commit of the iteration does not happen
+ * and the context stays usable.  -1 disarms.  Drops the captured graphs.
+ * Only iterations that run the persistent kernel (cllm_uses_persistent) are
+ * affected.  EINVAL on a null ctx, phase 0 or phase < -1.
+ */
+int cllm_test_hold_barrier(cllm_ctx *ctx, int phase);
+
+/*
+ * Allocation-failure injection: the k-th device (or pinned host) allocation
+ * the library makes from now on (k = 0: the next one) fails as if memory
+ * were exhausted; the call that made it returns CLLM_ENOMEM after releasing
+ * what it had allocated.  One-shot; k < 0 disarms.  Process-wide.
+ */
+void cllm_test_fail_alloc(int k);
+
 #ifdef __cplusplus
 }
 #endif

@@ -6,6 +6,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstring>
@@ -185,6 +186,7 @@ struct cllm_ctx {
   std::vector<std::string> last_phase_names;
   std::vector<unsigned long long> last_cta_stamps;
   int trace_phase = -1;  // profiling: phase whose MMA stage arrivals are traced
+  int hold_phase = -1;   // test hook: grid barrier that cannot open (bounded-wait path)
   std::map<std::tuple<int, int, int, int, int, unsigned long long, int, int, int, int>, GraphEntry>
       graphs;
   // profiling
@@ -207,11 +209,27 @@ int cuda_fail(cudaError_t e, const char* where) {
   return CLLM_ECUDA;
 }
 
+// Test hook (cllm_test_fail_alloc): the device or pinned allocation that
+// brings the countdown from 0 to -1 fails as if the memory were exhausted.
+std::atomic<int> g_alloc_countdown{-1};
+
+bool alloc_injected_failure() {
+  int v = g_alloc_countdown.load();
+  while (v >= 0 && !g_alloc_countdown.compare_exchange_weak(v, v - 1)) {
+  }
+  return v == 0;
+}
+
+cudaError_t lib_malloc(void** p, size_t bytes) {
+  if (alloc_injected_failure()) return cudaErrorMemoryAllocation;
+  return cudaMalloc(p, bytes);
+}
+
 template <typename T>
 bool dev_alloc(cllm_ctx* c, T** p, size_t bytes) {
   void* v = nullptr;
   if (bytes == 0) bytes = 16;
-  if (cudaMalloc(&v, bytes) != cudaSuccess) return false;
+  if (lib_malloc(&v, bytes) != cudaSuccess) return false;
   if (cudaMemset(v, 0, bytes) != cudaSuccess) return false;
   c->allocs.push_back(v);
   *p = static_cast<T*>(v);
@@ -675,7 +693,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   // device copies
   auto upload = [&](const void* src, size_t bytes) -> void* {
     void* p = nullptr;
-    if (cudaMalloc(&p, bytes) != cudaSuccess) return nullptr;
+    if (lib_malloc(&p, bytes) != cudaSuccess) return nullptr;
     ge.bufs.push_back(p);
     if (src && cudaMemcpy(p, src, bytes, cudaMemcpyHostToDevice) != cudaSuccess) return nullptr;
     if (!src && cudaMemset(p, 0, bytes) != cudaSuccess) return nullptr;
@@ -716,6 +734,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   sa.stamps = c->profiling ? ge.stamps : nullptr;
   sa.cta_stamps = c->profiling ? ge.cta_stamps : nullptr;
   sa.trace_phase = c->trace_phase;
+  sa.hold_phase = c->hold_phase;
   sa.err = c->err;
   return CLLM_OK;
 }
@@ -743,7 +762,8 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
   }
   cllm_ctx::GraphEntry ge;
   std::vector<int2> qt = step_qtiles(B, n);
-  if (cudaMalloc(&ge.qtiles, qt.size() * sizeof(int2)) != cudaSuccess) return CLLM_ENOMEM;
+  if (lib_malloc(reinterpret_cast<void**>(&ge.qtiles), qt.size() * sizeof(int2)) != cudaSuccess)
+    return CLLM_ENOMEM;
   if (cudaMemcpy(ge.qtiles, qt.data(), qt.size() * sizeof(int2), cudaMemcpyHostToDevice) !=
       cudaSuccess) {
     cudaFree(ge.qtiles);
@@ -1167,7 +1187,7 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
       rc = CLLM_ENOMEM;
       break;
     }
-    if (cudaMallocHost(&c->status_host, 32) != cudaSuccess) {
+    if (alloc_injected_failure() || cudaMallocHost(&c->status_host, 32) != cudaSuccess) {
       rc = CLLM_ENOMEM;
       break;
     }
@@ -1831,9 +1851,8 @@ extern "C" int cllm_test_phase_stamps(cllm_ctx* c, unsigned long long* out, int 
   return n;
 }
 
-extern "C" int cllm_test_set_trace_phase(cllm_ctx* c, int phase) {
-  if (!c) return CLLM_EINVAL;
-  c->trace_phase = phase;
+namespace {
+int drop_graphs(cllm_ctx* c) {
   cudaSetDevice(c->dev);
   if (cudaStreamSynchronize(c->stream) != cudaSuccess) return cuda_fail(cudaGetLastError(), "sync");
   for (auto& kv : c->graphs) {
@@ -1844,6 +1863,21 @@ extern "C" int cllm_test_set_trace_phase(cllm_ctx* c, int phase) {
   c->graphs.clear();
   return CLLM_OK;
 }
+}  // namespace
+
+extern "C" int cllm_test_set_trace_phase(cllm_ctx* c, int phase) {
+  if (!c) return CLLM_EINVAL;
+  c->trace_phase = phase;
+  return drop_graphs(c);
+}
+
+extern "C" int cllm_test_hold_barrier(cllm_ctx* c, int phase) {
+  if (!c || phase == 0 || phase < -1) return CLLM_EINVAL;
+  c->hold_phase = phase;
+  return drop_graphs(c);
+}
+
+extern "C" void cllm_test_fail_alloc(int k) { g_alloc_countdown.store(k < 0 ? -1 : k); }
 
 extern "C" int cllm_test_cta_stamps(cllm_ctx* c, unsigned long long* out, long long cap) {
   if (!c) return CLLM_EINVAL;

@@ -269,12 +269,12 @@ __device__ bool tc_produce(const TcPipe& P, int& idx, int& issued_b, const GemmA
     }
     open = dep.ready();
     if (open) break;
-    if (*P.abort) return false;
+    if (*P.abort) break;  // gave up: dep.wait below returns false at once
     if (t0 == 0) {
       t0 = globaltimer_ns();
     } else if (globaltimer_ns() - t0 > kWaitBudgetNs) {
       *P.abort = 1;
-      return false;
+      break;
     }
     __nanosleep(32);
   }

@@ -197,6 +197,9 @@ struct StepArgs {
   // arrivals (ns); then kTraceCap stage arrivals per CTA of phase trace_phase
   unsigned long long* cta_stamps;
   int trace_phase;  // -1: none
+  // test hook: the grid barrier before this phase waits for one arrival more
+  // than the grid makes, so its bounded waits run out (-1: none)
+  int hold_phase;
   int* err;
 };
 

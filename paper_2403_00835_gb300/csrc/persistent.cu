@@ -90,6 +90,12 @@ __device__ bool epilogue_phase(const TcPipe& P, int& acc, uint32_t& accph, const
   }
 }
 
+// Arrivals the grid barrier must count before phase p starts: every CTA
+// arrives once after each earlier phase.  (The hold hook asks for one more.)
+__device__ __forceinline__ unsigned barrier_target(const StepArgs& A, int p, int G) {
+  return static_cast<unsigned>(p) * static_cast<unsigned>(G) + (p == A.hold_phase ? 1u : 0u);
+}
+
 template <class Cfg>
 __device__ bool mma_phase(const TcPipe& P, int& idx, int& acc, uint32_t& accph, const PhaseDesc& ph,
                           int cta, unsigned long long* prof, long long prof_stride,
@@ -133,7 +139,7 @@ __global__ void __launch_bounds__(192, 1)
       for (int p = 0; p < A.n_phases; ++p) {
         const PhaseDesc& ph = A.phases[p];
         if (ph.kind != PH_GEMM) continue;
-        const GridDep dep{A.bar, static_cast<unsigned>(p) * static_cast<unsigned>(G)};
+        const GridDep dep{A.bar, barrier_target(A, p, G)};
         const size_t PG = static_cast<size_t>(A.n_phases) * G;
         unsigned long long* cs =
             A.cta_stamps != nullptr ? A.cta_stamps + static_cast<size_t>(p) * G + cta : nullptr;
@@ -178,7 +184,7 @@ __global__ void __launch_bounds__(192, 1)
       const int kind = ph.kind;
       if (kind == PH_ACCEPT && cta != 0) break;
       if (p > 0) {
-        const GridDep dep{A.bar, static_cast<unsigned>(p) * static_cast<unsigned>(G)};
+        const GridDep dep{A.bar, barrier_target(A, p, G)};
         if (r == 0) s_flag = dep.wait(P.abort) ? 1 : 0;
         sync();
         const bool ok = s_flag != 0;
