@@ -315,40 +315,54 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
     // HD/4 consecutive threads as float4 (coalesced)
     constexpr int TPR = HD / 4;     // threads per row
     constexpr int RPP = 128 / TPR;  // rows per pass
+    constexpr int NP = kQTile / RPP;  // passes
     const int d = (tid % TPR) * 4;
+    // all passes' shared-memory reads and arithmetic first, then the global
+    // stores: a store may not be reordered above a later pass's loads, so
+    // interleaving them would serialise the passes
+    float4 ov[NP];
+    float lsum[NP], Mrow[NP];
 #pragma unroll
-    for (int row = tid / TPR; row < kQTile; row += RPP) {
-      if (row < nr) {
-        float M = -INFINITY;
+    for (int k = 0; k < NP; ++k) {
+      const int row = tid / TPR + k * RPP;
+      float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
-        const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + rg;
-        float4 ov = make_float4(0.f, 0.f, 0.f, 0.f);
-        float l = 0.f;
-        if (M != -INFINITY) {
-          float f[4];
+      for (int w = 0; w < 4; ++w) M = fmaxf(M, sm.m[w][row]);
+      ov[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+      float l = 0.f;
+      if (row < nr && M != -INFINITY) {
+        float f[4];
 #pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            f[w] = exp2f(sm.m[w][row] - M);
-            l += f[w] * sm.l[w][row];
-          }
-          const float4 w0 = *reinterpret_cast<const float4*>(&co[0][row][d]);
-          const float4 w1 = *reinterpret_cast<const float4*>(&co[1][row][d]);
-          const float4 w2 = *reinterpret_cast<const float4*>(&co[2][row][d]);
-          const float4 w3 = *reinterpret_cast<const float4*>(&co[3][row][d]);
-          ov = make_float4(((f[0] * w0.x + f[1] * w1.x) + f[2] * w2.x) + f[3] * w3.x,
-                           ((f[0] * w0.y + f[1] * w1.y) + f[2] * w2.y) + f[3] * w3.y,
-                           ((f[0] * w0.z + f[1] * w1.z) + f[2] * w2.z) + f[3] * w3.z,
-                           ((f[0] * w0.w + f[1] * w1.w) + f[2] * w2.w) + f[3] * w3.w);
+        for (int w = 0; w < 4; ++w) {
+          f[w] = exp2f(sm.m[w][row] - M);
+          l += f[w] * sm.l[w][row];
         }
+        const float4 w0 = *reinterpret_cast<const float4*>(&co[0][row][d]);
+        const float4 w1 = *reinterpret_cast<const float4*>(&co[1][row][d]);
+        const float4 w2 = *reinterpret_cast<const float4*>(&co[2][row][d]);
+        const float4 w3 = *reinterpret_cast<const float4*>(&co[3][row][d]);
+        ov[k] = make_float4(((f[0] * w0.x + f[1] * w1.x) + f[2] * w2.x) + f[3] * w3.x,
+                            ((f[0] * w0.y + f[1] * w1.y) + f[2] * w2.y) + f[3] * w3.y,
+                            ((f[0] * w0.z + f[1] * w1.z) + f[2] * w2.z) + f[3] * w3.z,
+                            ((f[0] * w0.w + f[1] * w1.w) + f[2] * w2.w) + f[3] * w3.w);
+      }
+      lsum[k] = l;
+      Mrow[k] = M;
+    }
+#pragma unroll
+    for (int k = 0; k < NP; ++k) {
+      const int row = tid / TPR + k * RPP;
+      if (row < nr) {
         if (single) {
           // the tile's only range: the attention output itself
+          const float l = lsum[k];
           st_gin4(static_cast<__nv_bfloat16*>(a.out),
                   static_cast<size_t>(row_g0 + row) * a.H * HD + h * HD + d, a.plane_out,
-                  make_float4(ov.x / l, ov.y / l, ov.z / l, ov.w / l));
+                  make_float4(ov[k].x / l, ov[k].y / l, ov[k].z / l, ov[k].w / l));
         } else {
-          *reinterpret_cast<float4*>(a.part_o + pidx * HD + d) = ov;
-          if (d == 0) a.part_ml[pidx] = make_float2(M, l);
+          const size_t pidx = (static_cast<size_t>(row_g0 + row) * a.H + h) * a.nch_max + rg;
+          *reinterpret_cast<float4*>(a.part_o + pidx * HD + d) = ov[k];
+          if (d == 0) a.part_ml[pidx] = make_float2(Mrow[k], lsum[k]);
         }
       }
     }

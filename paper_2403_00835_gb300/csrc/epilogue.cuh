@@ -233,16 +233,28 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
       }
       epi_sync();
     }
+    using AT = typename AttnType<Act>::T;
+    if (sec == 0) {
 #pragma unroll
-    for (int j = 0; j < kEpiCols; ++j) {
-      const int t = t0 + j;
-      if (t >= e.T) continue;
-      using AT = typename AttnType<Act>::T;
-      if (sec == 0) {
-        st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
-      } else {
-        const int p = s.prepared ? s.pos_all[t] : e.pos[t];
-        const int b = s.prepared ? s.bidx_all[t] : e.bidx[t];
+      for (int j = 0; j < kEpiCols; ++j) {
+        const int t = t0 + j;
+        if (t < e.T) st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
+      }
+    } else {
+      // every column's cache row first: a load may not move above an
+      // earlier store, so reading them between the stores would serialise
+      int pj[kEpiCols], bj[kEpiCols];
+#pragma unroll
+      for (int j = 0; j < kEpiCols; ++j) {
+        const int t = min(t0 + j, e.T - 1);
+        pj[j] = s.prepared ? s.pos_all[t] : e.pos[t];
+        bj[j] = s.prepared ? s.bidx_all[t] : e.bidx[t];
+      }
+#pragma unroll
+      for (int j = 0; j < kEpiCols; ++j) {
+        const int t = t0 + j;
+        if (t >= e.T) continue;
+        const int p = pj[j], b = bj[j];
         if (p < 0 || p >= e.max_seq) {
           atomicOr(e.err, DERR_CAPACITY);
           continue;
@@ -263,13 +275,16 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
     if (r < 64) {
       const int f = mt * 64 + r;
       if (f < e.F) {
+        float up[kEpiCols];  // read before the stores (see the QKV case)
+#pragma unroll
+        for (int j = 0; j < kEpiCols; ++j) up[j] = s.x[j][r + 64];
 #pragma unroll
         for (int j = 0; j < kEpiCols; ++j) {
           const int t = t0 + j;
           if (t < e.T) {
-            const float gt = v[j], up = s.x[j][r + 64];
+            const float gt = v[j];
             st_gin(reinterpret_cast<Act*>(e.h_out), static_cast<size_t>(t) * e.F + f, e.plane_h,
-                   gt / (1.f + expf(-gt)) * up);
+                   gt / (1.f + expf(-gt)) * up[j]);
           }
         }
       }
