@@ -580,7 +580,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   const int T = B * n;
   const int NL = c->NL;
   const int mapB = 7 * NL + 1;
-  std::vector<CUtensorMap> maps(7 * NL + 4);
+  std::vector<CUtensorMap> maps(7 * NL + 7);
   for (int l = 0; l < NL; ++l) {
     const LayerW& L = c->layers[l];
     maps[7 * l + 0] = L.mq;
@@ -597,6 +597,13 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   if (!make_map(&maps[mapB], c->xg, c->d, rows, bn) ||
       !make_map(&maps[mapB + 1], c->attn, c->dq, rows, bn) ||
       !make_map(&maps[mapB + 2], c->h, c->F, rows, bn))
+    return CLLM_EINVAL;
+  // attention tiles: K/V caches of all layers as rows of hd values, Q rows
+  const int mapA = 7 * NL + 4;
+  const uint64_t kv_rows = static_cast<uint64_t>(NL) * c->layer_kv_elems / c->hd;
+  if (!make_map(&maps[mapA], c->kc, c->hd, kv_rows, kAttnChunk) ||
+      !make_map(&maps[mapA + 1], c->vc, c->hd, kv_rows, kAttnChunk) ||
+      !make_map(&maps[mapA + 2], c->q, c->dq, static_cast<uint64_t>(c->Tcap), kQTile))
     return CLLM_EINVAL;
 
   FwdSpec f{};
@@ -645,6 +652,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     at.kind = PH_ATTN;
     at.k_cache = kl;
     at.v_cache = vl;
+    at.kv_row0 = static_cast<int>(static_cast<size_t>(l) * c->layer_kv_elems / c->hd);
     ph.push_back(at);
     e = base_epi(c, T);
     e.x = c->x;
@@ -735,12 +743,17 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   sa.cta_stamps = c->profiling ? ge.cta_stamps : nullptr;
   sa.trace_phase = c->trace_phase;
   sa.hold_phase = c->hold_phase;
+  sa.map_attn_k = mapA;
+  sa.map_attn_v = mapA + 1;
+  sa.map_attn_q = mapA + 2;
   sa.err = c->err;
   return CLLM_OK;
 }
 
 bool persistent_ok(cllm_ctx* c, int B, int n) {
-  return c->bf16 && c->persistent && B * n <= 128 && 7 * c->NL + 4 <= kMaxStepMaps &&
+  // (the attention's K/V tensor maps address cache rows with 32-bit coordinates)
+  return c->bf16 && c->persistent && B * n <= 128 && 7 * c->NL + 7 <= kMaxStepMaps &&
+         static_cast<uint64_t>(c->NL) * c->layer_kv_elems / c->hd + kAttnChunk < (1ull << 31) &&
          B * ceil_div(n, kQTile) <= kMaxQTilesStep && (c->hd == 64 || c->hd == 128);
 }
 

@@ -19,6 +19,48 @@ struct AttnTileSmem {
   float l[4][kQTile];
 };
 
+// The same tile filled by TMA tensor-map loads (persistent kernel): Q, K and V
+// as 64-column halves of [rows][128 B] with the 128-byte swizzle (16-byte
+// chunk c of row r stored at chunk c ^ (r mod 8)), which keeps ldmatrix free
+// of bank conflicts without padding; one TMA operation moves a whole
+// 128-row half.  After the key loop K and V hold the warps' merge area.
+template <int HD>
+struct AttnTileSmemTma {
+  alignas(1024) uint8_t q[kQTile * HD * 2];
+  alignas(1024) uint8_t k[kAttnChunk * HD * 2];
+  alignas(1024) uint8_t v[kAttnChunk * HD * 2];
+  float m[4][kQTile];
+  float l[4][kQTile];
+  uint64_t bar[2];  // completion of the K (with Q) and V loads; fresh per work item
+};
+
+// Tensor maps of the TMA tile loads: the K and V caches of all layers as
+// [layer][b][kv_head][pos] rows of hd fp16 values (boxes of 128 rows x 64
+// columns), Q as [row][n_heads*hd] (boxes of 16 rows x 64 columns); kv_row0 =
+// the first row of this layer.
+struct AttnTma {
+  const CUtensorMap* k;
+  const CUtensorMap* v;
+  const CUtensorMap* q;
+  int kv_row0;
+};
+
+template <class T>
+struct IsTmaTile {
+  static constexpr bool value = false;
+};
+template <int HD>
+struct IsTmaTile<AttnTileSmemTma<HD>> {
+  static constexpr bool value = true;
+};
+
+// Byte address of 16-byte chunk `chunk` of row `row` in a swizzled tile of
+// `rows` rows per 64-column half.
+__device__ __forceinline__ uint32_t sw128_addr(uint32_t base, int rows, int row, int chunk) {
+  return base + static_cast<uint32_t>((chunk >> 3) * rows * 128 + row * 128 +
+                                      (((chunk & 7) ^ (row & 7)) << 4));
+}
+
 // Where the iteration's query-tile and sequence metadata are read from: the
 // kernel arguments (global memory), or a shared-memory copy made once per
 // phase (AttnMetaSmem) so that work items do not chain dependent loads.
@@ -126,15 +168,16 @@ __device__ __forceinline__ int attn_tile_ranges(const AttnArgs& a, const Meta& m
 // otherwise the range's partial (O, m, l) goes to slot `range` of the
 // partials (merged by the combine, which gives the same bits for one range).
 // Returns the tile index and head in qi_out, h_out.
-template <int HD, class Sync, class Meta = GlobalMeta>
-__device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnTileSmem<HD>& sm,
-                              int tid, Sync sync, int& qi_out, int& h_out, const Meta& md,
-                              bool direct_ok = true) {
+template <int HD, class Sync, class Meta = GlobalMeta, class Tile = AttnTileSmem<HD>>
+__device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, Tile& sm, int tid,
+                              Sync sync, int& qi_out, int& h_out, const Meta& md,
+                              bool direct_ok = true, const AttnTma* tma = nullptr) {
+  constexpr bool kTma = IsTmaTile<Tile>::value;
   // merge area: rows padded by 8 floats, so that the 8 row groups of a warp's
   // accumulator fragment fall in distinct banks
   constexpr int CLD = HD + 8;
-  static_assert(sizeof(float) * 4 * kQTile * CLD <= sizeof(__half) * kAttnChunk * (HD + 8),
-                "merge area must fit in the K tile");
+  static_assert(sizeof(float) * 4 * kQTile * CLD <= (kTma ? 2 : 1) * sizeof(sm.k),
+                "merge area must fit in the K (and V) tile");
   const int warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, cq = lane & 3;
   const int group = a.H / a.Hkv;
@@ -142,7 +185,7 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   const __half* Q = static_cast<const __half*>(a.q);
   const __half* KC = static_cast<const __half*>(a.k_cache);
   const __half* VC = static_cast<const __half*>(a.v_cache);
-  float (*co)[kQTile][CLD] = reinterpret_cast<float (*)[kQTile][CLD]>(&sm.k[0][0]);
+  float (*co)[kQTile][CLD] = reinterpret_cast<float (*)[kQTile][CLD]>(&sm.k[0]);
   const int qi = attn_find_qtile(pre, a.n_qtiles, item);
   const int local = item - pre[qi];
   const int rg = local / a.H, h = local - rg * a.H;
@@ -160,8 +203,14 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   const int kvh = h / group;
   const size_t kvbase = ((static_cast<size_t>(b) * a.Hkv + kvh) * a.max_seq) * HD;
   constexpr int CPR = HD * 2 / 16;  // 16-byte pieces per row
+  constexpr int NHALF = HD / 64;     // 64-column halves of a row (TMA boxes per tile)
+  uint64_t* barK = nullptr;
+  uint64_t* barV = nullptr;
+  uint32_t phK = 0, phV = 0;
+  int kvrow = 0;
 
-  auto load_kv = [&](__half (*dstm)[HD + 8], const __half* src, int c) {
+  // cp.async path: per-thread 16-byte copies, zero rows past the tile's keys
+  auto load_kv = [&](auto* dstm, const __half* src, int c) {
     const int kb = c * kAttnChunk;
     for (int i = tid; i < kAttnChunk * CPR; i += 128) {
       const int rr = i / CPR, pc = i - rr * CPR;
@@ -172,20 +221,59 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
         *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
     }
   };
+  // TMA path: one thread posts the byte count and issues a box per 64-column
+  // half.  Rows past the tile's keys hold other positions' (finite) cache
+  // values or the map's zero fill: their scores are masked to -inf, so their
+  // probabilities are exactly 0.
+  auto tma_kv = [&](uint8_t* dst, const CUtensorMap* map, int c, uint64_t* bar, bool with_q) {
+    if (tid == 0) {
+      mbar_arrive_expect_tx(bar, (with_q ? NHALF * kQTile * 128 : 0) + NHALF * kAttnChunk * 128);
+      if (with_q)
+        for (int hh = 0; hh < NHALF; ++hh)
+          tma_load_2d_nohint(sm.q + hh * kQTile * 128, tma->q, bar, h * HD + hh * 64, row_g0);
+      for (int hh = 0; hh < NHALF; ++hh)
+        tma_load_2d_nohint(dst + hh * kAttnChunk * 128, map, bar, hh * 64,
+                           kvrow + c * kAttnChunk);
+    }
+  };
+  auto wait_buf = [&](uint64_t* bar, uint32_t& ph) {
+    if (!mbar_wait(bar, ph & 1u, nullptr) && tid == 0) atomicOr(a.err, DERR_TIMEOUT);
+    ++ph;
+  };
 
-  // ---- Q (16 rows) and the first chunk's K: group 1; its V: group 2 ----
-  for (int i = tid; i < kQTile * CPR; i += 128) {
-    const int rr = i / CPR, pc = i - rr * CPR;
-    void* dst = &sm.q[rr][pc * 8];
-    if (rr < nr)
-      cp_async16(dst, Q + static_cast<size_t>(row_g0 + rr) * ldq + h * HD + pc * 8);
-    else
-      *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+  if constexpr (kTma) {
+    barK = &sm.bar[0];
+    barV = &sm.bar[1];
+    kvrow = tma->kv_row0 + (b * a.Hkv + kvh) * a.max_seq;
+    // fresh barrier phases per work item; every earlier generic write to this
+    // shared memory (merge area, GEMM epilogue) ordered before the TMA writes
+    fence_proxy_async_smem();
+    if (tid == 0) {
+      mbar_init(barK, 1);
+      mbar_init(barV, 1);
+      fence_mbar_init();
+    }
+    sync();
+    // ---- Q (16 rows) with the first chunk's K on barK; its V on barV ----
+    tma_kv(sm.k, tma->k, c0, barK, true);
+    tma_kv(sm.v, tma->v, c0, barV, false);
+  } else {
+    // ---- Q (16 rows) and the first chunk's K: group 1; its V: group 2 ----
+    for (int i = tid; i < kQTile * CPR; i += 128) {
+      const int rr = i / CPR, pc = i - rr * CPR;
+      void* dst = &sm.q[rr][pc * 8];
+      if (rr < nr)
+        cp_async16(dst, Q + static_cast<size_t>(row_g0 + rr) * ldq + h * HD + pc * 8);
+      else
+        *reinterpret_cast<uint4*>(dst) = make_uint4(0, 0, 0, 0);
+    }
+    load_kv(sm.k, KC, c0);
+    cp_async_commit();
+    load_kv(sm.v, VC, c0);
+    cp_async_commit();
   }
-  load_kv(sm.k, KC, c0);
-  cp_async_commit();
-  load_kv(sm.v, VC, c0);
-  cp_async_commit();
+  (void)phK;
+  (void)phV;
 
   const int wk0 = warp * 32;  // first key of this warp within a chunk
   const int posA = pos0 + g, posB = pos0 + g + 8;
@@ -196,8 +284,12 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
   float mA = -INFINITY, mB = -INFINITY, lA = 0.f, lB = 0.f;
   for (int c = c0; c < c1; ++c) {
     const int kb = c * kAttnChunk;
-    cp_async_wait_but1();  // Q and this chunk's K
-    sync();
+    if constexpr (kTma) {
+      wait_buf(barK, phK);  // (Q and) this chunk's K: TMA writes, seen by every waiter
+    } else {
+      cp_async_wait_but1();  // Q and this chunk's K
+      sync();
+    }
     float sc[4][4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
@@ -206,21 +298,35 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
 #pragma unroll
       for (int ks = 0; ks < HD / 16; ks += 2) {
         uint32_t qa0[4], qa1[4];
-        ldmatrix_x4(qa0, &sm.q[lane & 15][ks * 16 + (lane >> 4) * 8]);
-        ldmatrix_x4(qa1, &sm.q[lane & 15][(ks + 1) * 16 + (lane >> 4) * 8]);
+        if constexpr (kTma) {
+          const uint32_t qb = smem_u32(sm.q);
+          ldmatrix_x4_a(qa0, sw128_addr(qb, kQTile, lane & 15, ks * 2 + (lane >> 4)));
+          ldmatrix_x4_a(qa1, sw128_addr(qb, kQTile, lane & 15, (ks + 1) * 2 + (lane >> 4)));
+        } else {
+          ldmatrix_x4(qa0, &sm.q[lane & 15][ks * 16 + (lane >> 4) * 8]);
+          ldmatrix_x4(qa1, &sm.q[lane & 15][(ks + 1) * 16 + (lane >> 4) * 8]);
+        }
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           uint32_t kb4[4];
           const int mi = lane >> 3;
-          ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
+          if constexpr (kTma)
+            ldmatrix_x4_a(kb4, sw128_addr(smem_u32(sm.k), kAttnChunk, wk0 + 8 * j + (lane & 7),
+                                          (ks + (mi >> 1)) * 2 + (mi & 1)));
+          else
+            ldmatrix_x4(kb4, &sm.k[wk0 + 8 * j + (lane & 7)][(ks + (mi >> 1)) * 16 + (mi & 1) * 8]);
           mma_f16_16816(sc[j], qa0, kb4[0], kb4[1]);
           mma_f16_16816(sc[j], qa1, kb4[2], kb4[3]);
         }
       }
     }
     sync();  // every warp is done with K
-    if (c + 1 < c1) load_kv(sm.k, KC, c + 1);
-    cp_async_commit();  // (possibly empty) group: the next chunk's K
+    if constexpr (kTma) {
+      if (c + 1 < c1) tma_kv(sm.k, tma->k, c + 1, barK, false);
+    } else {
+      if (c + 1 < c1) load_kv(sm.k, KC, c + 1);
+      cp_async_commit();  // (possibly empty) group: the next chunk's K
+    }
     if (live) {
       // mask + scale (log2 domain), online softmax over the range's chunks
       float nA = mA, nB = mB;
@@ -269,8 +375,12 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
         o[dn][2] *= fB;
         o[dn][3] *= fB;
       }
-      cp_async_wait_but1();  // this chunk's V (the next K may be in flight)
-      sync();
+      if constexpr (kTma) {
+        wait_buf(barV, phV);  // this chunk's V (the next K may be in flight)
+      } else {
+        cp_async_wait_but1();  // this chunk's V (the next K may be in flight)
+        sync();
+      }
       // O += P V: A fragments of P for keys 16kk..16kk+15 are the S
       // accumulators of n-tiles 2kk, 2kk+1 (a0: row g keys 2c.., a1: row g+8,
       // a2/a3: +8 keys).
@@ -281,20 +391,32 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
         for (int dn = 0; dn < HD / 8; dn += 2) {
           uint32_t vb[4];
           const int mi = lane >> 3;
-          ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
+          if constexpr (kTma)
+            ldmatrix_x4_trans_a(vb, sw128_addr(smem_u32(sm.v), kAttnChunk,
+                                               wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7), dn + (mi >> 1)));
+          else
+            ldmatrix_x4_trans(vb, &sm.v[wk0 + 16 * kk + (mi & 1) * 8 + (lane & 7)][(dn + (mi >> 1)) * 8]);
           mma_f16_16816(o[dn], af, vb[0], vb[1]);
           mma_f16_16816(o[dn + 1], af, vb[2], vb[3]);
         }
       }
     } else {
-      cp_async_wait_but1();
-      sync();
+      if constexpr (kTma) {
+        wait_buf(barV, phV);
+      } else {
+        cp_async_wait_but1();
+        sync();
+      }
     }
     sync();  // every warp is done with V
-    if (c + 1 < c1) load_kv(sm.v, VC, c + 1);
-    cp_async_commit();  // (possibly empty) group: the next chunk's V
+    if constexpr (kTma) {
+      if (c + 1 < c1) tma_kv(sm.v, tma->v, c + 1, barV, false);
+    } else {
+      if (c + 1 < c1) load_kv(sm.v, VC, c + 1);
+      cp_async_commit();  // (possibly empty) group: the next chunk's V
+    }
   }
-  cp_async_wait_all();
+  if constexpr (!kTma) cp_async_wait_all();
   sync();
 #pragma unroll
   for (int dn = 0; dn < HD / 8; ++dn) {
@@ -368,6 +490,12 @@ __device__ bool attn_mma_item(const AttnArgs& a, int item, const int* pre, AttnT
     }
   }
   sync();
+  if constexpr (kTma) {
+    if (tid == 0) {  // every load of the item has been waited for
+      mbar_inval(barK);
+      mbar_inval(barV);
+    }
+  }
   qi_out = qi;
   h_out = h;
   return single;

@@ -180,6 +180,7 @@ struct PhaseDesc {
   EpiArgs e;
   const void* k_cache;
   const void* v_cache;
+  int kv_row0;  // attention: the layer's first row in the K/V cache tensor maps
 };
 
 struct StepArgs {
@@ -200,6 +201,8 @@ struct StepArgs {
   // test hook: the grid barrier before this phase waits for one arrival more
   // than the grid makes, so its bounded waits run out (-1: none)
   int hold_phase;
+  // attention tile loads: indices of the K-cache, V-cache and Q tensor maps
+  int map_attn_k, map_attn_v, map_attn_q;
   int* err;
 };
 
@@ -209,12 +212,14 @@ constexpr int kMaxQTilesStep = 256;  // query tiles of one iteration (persistent
 
 // Tensor maps travel by value in the kernel's parameter space (TMA reads
 // descriptors there as it does for per-GEMM kernels): 7 per layer + the LM
-// head + 3 activation maps, at most 32 layers (29 KB of the 32 KB limit).
-constexpr int kMaxStepMaps = 7 * 32 + 4;
+// head + 3 activation maps + the attention's K, V and Q maps, at most 32
+// layers (29.6 KB of the 32 KB limit).
+constexpr int kMaxStepMaps = 7 * 32 + 7;
 struct StepParams {
   StepArgs a;
   CUtensorMap maps[kMaxStepMaps];
 };
+static_assert(sizeof(StepParams) <= 32764, "kernel parameter space");
 
 // Launch of the persistent kernel (bn_max 32/64/128, head_dim 64/128).
 cudaError_t launch_step_persistent(const StepParams& p, int bn_max, int hd, int grid,

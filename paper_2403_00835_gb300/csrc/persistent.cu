@@ -27,7 +27,7 @@ __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + 
 
 template <int BNMAX, int HD>
 struct PersistCfg {
-  static constexpr size_t ATTN_BYTES = align_up(sizeof(AttnTileSmem<HD>), 16);
+  static constexpr size_t ATTN_BYTES = align_up(sizeof(AttnTileSmemTma<HD>), 1024);
   // the GEMM epilogue's part of the union: EpiSmem, then split-K staging
   // blocks (at least 4; as many as fit beside the attention tile)
   static constexpr size_t EPI_BYTES = align_up(sizeof(EpiSmem), 16);
@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(192, 1)
       reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* uni = base + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES;
   EpiSmem& es = *reinterpret_cast<EpiSmem*>(uni);
-  AttnTileSmem<HD>& at = *reinterpret_cast<AttnTileSmem<HD>*>(uni);
+  AttnTileSmemTma<HD>& at = *reinterpret_cast<AttnTileSmemTma<HD>*>(uni);  // 1024-aligned
   int* pre = reinterpret_cast<int*>(uni + PC::UNION);
   AttnMetaSmem& meta = *reinterpret_cast<AttnMetaSmem*>(uni + PC::UNION + PC::PRE_BYTES);
   uint8_t* bars = uni + PC::UNION + PC::META_BYTES;
@@ -220,9 +220,12 @@ __global__ void __launch_bounds__(192, 1)
           attn_total = attn_item_prefix(a, pre, r, sync, md);
         }
         const int total = attn_total;
+        const AttnTma tma{PRM.maps + A.map_attn_k, PRM.maps + A.map_attn_v, PRM.maps + A.map_attn_q,
+                          ph.kv_row0};
         for (int item = cta; item < total; item += G) {
           int qi, h;
-          if (attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md)) continue;  // output written
+          if (attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md, true, &tma))
+            continue;  // output written
           // the last range of (tile, head) to finish merges the tile's ranges
           sync();
           if (r == 0) {
