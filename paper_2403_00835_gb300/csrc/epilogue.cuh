@@ -7,6 +7,7 @@
 //   EPI_ARGMAX : x rms-scale, per-tile (max, argmax, 2nd max) of the logits;
 //                the last tile to finish reduces them to argmax and top-2 gap
 #pragma once
+#include <type_traits>
 #include <float.h>
 #include <limits.h>
 
@@ -202,6 +203,10 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
                           EpiSmem& s, const EpiPre* pre = nullptr) {
   const bool use_pre = pre != nullptr && pre->ok && pre->t0 == t0;
   const int lane = r & 31, grp = r >> 5;
+  // Every 16-column chunk but a ragged last one is full: its loops run
+  // without per-column guards (the epilogue warps run one per scheduler, so
+  // each branch and dependent step is exposed latency).
+  const bool full = t0 + kEpiCols <= e.T;
   if (KIND == EPI_QKV) {
     epi_norm_scale(e, t0, r, s);
     const int m = mt * kBM + r;
@@ -214,35 +219,45 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
 #pragma unroll
       for (int j = 0; j < kEpiCols; ++j) s.x[j][r] = v[j];
       epi_sync();
-      const int rp = (i < half) ? r + half : r - half;
-      const int fi = (i < half) ? i : i - half;
+      // rotate-half RoPE: v' = v cos + sgn * partner sin, sgn = -1 in the
+      // first half of the head
+      const bool lowhalf = i < half;
+      const int rp = lowhalf ? r + half : r - half;
+      const int fi = lowhalf ? i : i - half;
+      float cs_c[kEpiCols], cs_s[kEpiCols], pv[kEpiCols];
 #pragma unroll
       for (int j = 0; j < kEpiCols; ++j) {
-        const int t = t0 + j;
-        if (t < e.T) {
-          float2 cs;
-          if (use_pre) {
-            cs = make_float2(pre->a[j], pre->b[j]);
-          } else {
-            const int p = min(s.prepared ? s.pos_all[t] : e.pos[t], e.max_seq - 1);
-            cs = e.rope[static_cast<size_t>(p) * half + fi];
-          }
-          const float pv = s.x[j][rp];
-          v[j] = (i < half) ? (v[j] * cs.x - pv * cs.y) : (v[j] * cs.x + pv * cs.y);
+        const int t = min(t0 + j, e.T - 1);
+        if (use_pre) {
+          cs_c[j] = pre->a[j];
+          cs_s[j] = pre->b[j];
+        } else {
+          const int p = min(s.prepared ? s.pos_all[t] : e.pos[t], e.max_seq - 1);
+          const float2 cs = e.rope[static_cast<size_t>(p) * half + fi];
+          cs_c[j] = cs.x;
+          cs_s[j] = cs.y;
         }
+        pv[j] = s.x[j][rp];
+      }
+#pragma unroll
+      for (int j = 0; j < kEpiCols; ++j) {
+        const float ps = pv[j] * cs_s[j];
+        v[j] = lowhalf ? (v[j] * cs_c[j] - ps) : (v[j] * cs_c[j] + ps);
       }
       epi_sync();
     }
     using AT = typename AttnType<Act>::T;
     if (sec == 0) {
+      AT* q = reinterpret_cast<AT*>(e.q_out) + static_cast<size_t>(t0) * e.dq + m;
 #pragma unroll
-      for (int j = 0; j < kEpiCols; ++j) {
-        const int t = t0 + j;
-        if (t < e.T) st_act(reinterpret_cast<AT*>(e.q_out), static_cast<size_t>(t) * e.dq + m, v[j]);
-      }
+      for (int j = 0; j < kEpiCols; ++j)
+        if (full || t0 + j < e.T) st_act(q, static_cast<size_t>(j) * e.dq, v[j]);
     } else {
       // every column's cache row first: a load may not move above an
       // earlier store, so reading them between the stores would serialise
+      AT* cache = reinterpret_cast<AT*>(sec == 1 ? e.k_cache : e.v_cache) +
+                  static_cast<size_t>(head) * e.max_seq * e.hd + i;
+      const size_t bstride = static_cast<size_t>(e.n_kv_heads) * e.max_seq * e.hd;
       int pj[kEpiCols], bj[kEpiCols];
 #pragma unroll
       for (int j = 0; j < kEpiCols; ++j) {
@@ -250,19 +265,17 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
         pj[j] = s.prepared ? s.pos_all[t] : e.pos[t];
         bj[j] = s.prepared ? s.bidx_all[t] : e.bidx[t];
       }
+      bool bad = false;
 #pragma unroll
       for (int j = 0; j < kEpiCols; ++j) {
-        const int t = t0 + j;
-        if (t >= e.T) continue;
-        const int p = pj[j], b = bj[j];
-        if (p < 0 || p >= e.max_seq) {
-          atomicOr(e.err, DERR_CAPACITY);
-          continue;
-        }
-        const size_t off =
-            ((static_cast<size_t>(b) * e.n_kv_heads + head) * e.max_seq + p) * e.hd + i;
-        st_act(reinterpret_cast<AT*>(sec == 1 ? e.k_cache : e.v_cache), off, v[j]);
+        const bool live = full || t0 + j < e.T;
+        const bool inside = static_cast<unsigned>(pj[j]) < static_cast<unsigned>(e.max_seq);
+        if (live && inside)
+          st_act(cache, static_cast<size_t>(bj[j]) * bstride + static_cast<size_t>(pj[j]) * e.hd,
+                 v[j]);
+        bad |= live && !inside;
       }
+      if (bad) atomicOr(e.err, DERR_CAPACITY);
     }
   } else if (KIND == EPI_GATEUP) {
     epi_norm_scale(e, t0, r, s);
@@ -275,37 +288,43 @@ __device__ void epi_apply(const EpiArgs& e, int mt, int t0, float (&v)[kEpiCols]
     if (r < 64) {
       const int f = mt * 64 + r;
       if (f < e.F) {
-        float up[kEpiCols];  // read before the stores (see the QKV case)
-#pragma unroll
-        for (int j = 0; j < kEpiCols; ++j) up[j] = s.x[j][r + 64];
+        float h[kEpiCols];  // SwiGLU of every column first, then the stores
 #pragma unroll
         for (int j = 0; j < kEpiCols; ++j) {
-          const int t = t0 + j;
-          if (t < e.T) {
-            const float gt = v[j];
-            st_gin(reinterpret_cast<Act*>(e.h_out), static_cast<size_t>(t) * e.F + f, e.plane_h,
-                   gt / (1.f + expf(-gt)) * up[j]);
-          }
+          const float gt = v[j], up = s.x[j][r + 64];
+          if constexpr (std::is_same<Act, float>::value)
+            h[j] = gt / (1.f + expf(-gt)) * up;
+          else  // bf16 engine: the fast intrinsics' error is far below the lo plane's
+            h[j] = __fdividef(gt, 1.f + __expf(-gt)) * up;
         }
+        Act* hp = reinterpret_cast<Act*>(e.h_out) + static_cast<size_t>(t0) * e.F + f;
+#pragma unroll
+        for (int j = 0; j < kEpiCols; ++j)
+          if (full || t0 + j < e.T) st_gin(hp, static_cast<size_t>(j) * e.F, e.plane_h, h[j]);
       }
     }
     epi_sync();
   } else if (KIND == EPI_RESID) {
     const int m = mt * kBM + r;
     const float gn = use_pre ? pre->g : ld_act(reinterpret_cast<const Act*>(e.gnext), m);
-    float sq[kEpiCols];
+    float* xp = e.x + static_cast<size_t>(t0) * e.d + m;
+    Act* gp = reinterpret_cast<Act*>(e.xg) + static_cast<size_t>(t0) * e.d + m;
+    float xi[kEpiCols], sq[kEpiCols];
 #pragma unroll
     for (int j = 0; j < kEpiCols; ++j) {
-      const int t = t0 + j;
-      sq[j] = 0.f;
-      if (t < e.T) {
-        const size_t o = static_cast<size_t>(t) * e.d + m;
-        // L2 read: other CTAs rewrite the residual stream in earlier phases
-        // of the persistent kernel, and L1 is not coherent across SMs
-        const float xi = (use_pre ? pre->a[j] : __ldcg(e.x + o)) + v[j];
-        e.x[o] = xi;
-        st_gin(reinterpret_cast<Act*>(e.xg), o, e.plane_x, xi * gn);
-        sq[j] = xi * xi;
+      const bool live = full || t0 + j < e.T;
+      // L2 read: other CTAs rewrite the residual stream in earlier phases
+      // of the persistent kernel, and L1 is not coherent across SMs
+      const float x0 = use_pre ? pre->a[j] : (live ? __ldcg(xp + static_cast<size_t>(j) * e.d) : 0.f);
+      xi[j] = x0 + v[j];
+      sq[j] = live ? xi[j] * xi[j] : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < kEpiCols; ++j) {
+      if (full || t0 + j < e.T) {
+        const size_t o = static_cast<size_t>(j) * e.d;
+        xp[o] = xi[j];
+        st_gin(gp, o, e.plane_x, xi[j] * gn);
       }
     }
     const float col = warp_colsum16(sq, lane);
