@@ -51,6 +51,10 @@ constexpr size_t solo_smem_bytes() {
   return 1024 + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES + sizeof(EpiSmem) + 16 +
          kSoloRedSlots * kRedSlotBytes + tc_bar_bytes(Cfg::STAGES);
 }
+constexpr size_t kSmemLimit = 227 * 1024 - 256;  // minus static shared memory
+static_assert(solo_smem_bytes<32>() <= kSmemLimit && solo_smem_bytes<64>() <= kSmemLimit &&
+                  solo_smem_bytes<128>() <= kSmemLimit && solo_smem_bytes<256>() <= kSmemLimit,
+              "per-GEMM kernel shared memory over the 227 KB limit");
 
 template <int KIND, int BNMAX>
 __global__ void __launch_bounds__(192, 1)

@@ -39,7 +39,7 @@ struct PersistCfg {
   static constexpr size_t PRE_BYTES = align_up(4 * (kMaxQTilesStep + 1), 16);
   static constexpr size_t META_BYTES = PRE_BYTES + align_up(sizeof(AttnMetaSmem), 16);
   static constexpr int STAGE_BYTES = kBM * kBK * 2 + 2 * BNMAX * kBK * 2;
-  static constexpr size_t BUDGET = 227 * 1024;
+  static constexpr size_t BUDGET = 227 * 1024 - 256;  // minus the kernel's static shared memory
   static constexpr size_t FIXED = 1024 + UNION + META_BYTES + tc_bar_bytes(8) + 64;
   static constexpr int FIT = static_cast<int>((BUDGET - FIXED) / STAGE_BYTES);
   static constexpr int STAGES = FIT > 8 ? 8 : FIT;
