@@ -91,6 +91,19 @@ int cllm_test_hold_barrier(cllm_ctx *ctx, int phase);
  */
 void cllm_test_fail_alloc(int k);
 
+/*
+ * Host-only (no CUDA call): the work split of one weight-GEMM launch of
+ * `mtiles` 128-row weight tiles over K (inner dimension) for T token columns
+ * on `sms` SMs, as the library plans it.  out[8] = {mtiles, ntiles (token
+ * tiles), kchunks (64-column chunks of K), cpc (chunks per CTA), bn (token
+ * columns of a tile), bn_max (kernel variant), maxc (most CTAs sharing one
+ * tile), grid (CTAs)}.  T <= 256: one token tile and the (tile, chunk) space
+ * cut into equal contiguous ranges that depend on the weight shape and the SM
+ * count only; T > 256: whole 128 x 256 tiles per CTA.  EINVAL on a null out
+ * or a non-positive argument.
+ */
+int cllm_test_plan_gemm(int mtiles, int K, int T, int sms, int *out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -1892,6 +1892,14 @@ extern "C" int cllm_test_hold_barrier(cllm_ctx* c, int phase) {
 
 extern "C" void cllm_test_fail_alloc(int k) { g_alloc_countdown.store(k < 0 ? -1 : k); }
 
+extern "C" int cllm_test_plan_gemm(int mtiles, int K, int T, int sms, int* out) {
+  if (!out || mtiles < 1 || K < 1 || T < 1 || sms < 1) return CLLM_EINVAL;
+  const Part p = plan_gemm(mtiles, K, T, sms);
+  const int v[8] = {p.mtiles, p.ntiles, p.kchunks, p.cpc, p.bn, p.bn_max, p.maxc, p.grid};
+  for (int i = 0; i < 8; ++i) out[i] = v[i];
+  return CLLM_OK;
+}
+
 extern "C" int cllm_test_cta_stamps(cllm_ctx* c, unsigned long long* out, long long cap) {
   if (!c) return CLLM_EINVAL;
   const long long n = static_cast<long long>(c->last_cta_stamps.size());
