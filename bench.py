@@ -113,6 +113,21 @@ def dist_setup():
     return world, rank, local
 
 
+def rank_aggregate(dist, device, elapsed, count):
+    """Whole-job numbers of a replicas-only run (every rank decodes its own
+    sequences, nothing is exchanged on the data path): the slowest rank's
+    elapsed time and the sum of the ranks' counts.  Single process (dist is
+    None): unchanged."""
+    if dist is None:
+        return float(elapsed), float(count)
+    import torch
+    t = torch.tensor([float(elapsed)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    c = torch.tensor([float(count)], device=device, dtype=torch.float64)
+    dist.all_reduce(c)
+    return float(t.item()), float(c.item())
+
+
 # Table 3's fast-forwarded token counts (accepted tokens per iteration,
 # including the head) of the CLLMs, per n-token length and dataset.  The step
 # time does not depend on acceptance, so tokens/s at the paper's acceptance is
@@ -306,13 +321,7 @@ def run_ours(args, world, rank, local):
         ev1.record(stream)
         torch.cuda.synchronize()
         ms = ev0.elapsed_time(ev1)
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-            cc = torch.tensor([committed], device="cuda", dtype=torch.float64)
-            dist.all_reduce(cc)
-            committed = float(cc.item())
+        ms, committed = rank_aggregate(dist, "cuda", ms, committed)
         return ms, committed, restarts
 
     # Jacobi (n) and the same-kernel AR baseline (n = 1)
@@ -334,10 +343,13 @@ def run_ours(args, world, rank, local):
 
     # end to end through the C ABI with host buffers (prefill + decode + copies)
     torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
     t0 = time.perf_counter()
     out, iters = eng.jacobi_decode(prompts, n, max_new, seed=2)
     e2e_s = time.perf_counter() - t0
-    e2e_val = float(np.sum(out >= 0)) * world / e2e_s
+    e2e_s, e2e_tokens = rank_aggregate(dist, "cuda", e2e_s, int(np.sum(out >= 0)))
+    e2e_val = e2e_tokens / e2e_s
     e2e_iters = max(1, int(np.max(iters)))
     # host<->device bytes of that call, per decode iteration: the prompt
     # tokens and lengths in, the status word (12 bytes) out every iteration,
