@@ -54,3 +54,20 @@ def test_create_rejects_null_arguments(lib):
 
 def test_library_is_in_tree():
     assert cllm.library_path().startswith(os.path.join(ROOT, "paper_2403_00835_gb300"))
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """No CPU fallback: without the built library the binding raises."""
+    monkeypatch.setattr(cllm, "_lib", None)
+    monkeypatch.setattr(cllm._build, "LIB", str(tmp_path / "absent" / "libcllm.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        cllm.load(build_if_missing=False)
+
+
+def test_engine_rejects_host_weights():
+    """The engine takes device weights only (PyTorch supplies memory, never compute)."""
+    torch = pytest.importorskip("torch")
+    from paper_2403_00835_gb300 import synthetic as syn
+    w = syn.make_weights(syn.TINY, seed=0, device="cpu")
+    with pytest.raises(ValueError, match="CUDA"):
+        cllm.Engine(syn.TINY, w, max_batch=1, max_seq=64, max_block=8)
