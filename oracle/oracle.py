@@ -23,7 +23,7 @@ Layout
         ``jacobi_vanilla``  Eq. 3 iterated without any cache until
                             y^(k) = y^(k-1) (Sec. 3.1), used only as a pin.
 
-Readings of the paper this oracle takes (each also listed in the design doc):
+Readings of the paper this oracle takes:
   * The first block token is the head: the prediction from the committed
     context, correct by construction (Alg. 3's y_0 from the prefill).  The
     accepted count of a step is a = 1 + the number of leading positions k >= 1
