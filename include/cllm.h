@@ -142,6 +142,9 @@ int cllm_prefill(cllm_ctx *ctx, int B, const int32_t *tokens, const int32_t *len
  * Outputs (host): next_out[B][n] = P (y^(j+1) shifted: P[k] predicts block
  * position k+1), accepted_out[B] = a_b; gap_out[B][n] or NULL; logits_out
  * [B][n][vocab] fp32 or NULL (debug: logits are otherwise never stored).
+ * The step runs the kernel(s) the decode loop runs for this shape (the
+ * persistent per-iteration kernel where cllm_uses_persistent(ctx, n) holds);
+ * with logits_out that kernel's LM-head phase also stores the logits.
  * Errors: EINVAL (n outside [1, max_block], token outside the vocab),
  * ESTATE (no prefill), ECAPACITY (L_b + n > max_seq), ECUDA, EDEVICE, ETIMEOUT.
  */

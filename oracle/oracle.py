@@ -329,6 +329,7 @@ class DecodeResult:
     min_gap: list = field(default_factory=list)    # per iteration: min gap over the committed rows' predictions
     min_gap_all: list = field(default_factory=list)  # per iteration: min gap over every row of the block
     trajectory: list = field(default_factory=list)  # blocks fed to each iteration
+    steps: list = field(default_factory=list)  # StepResult of each iteration (keep_steps)
 
 
 def ar_decode(model: OracleModel, prompt: Sequence[int], max_new: int, eos_id: int = -1) -> DecodeResult:
@@ -353,14 +354,16 @@ def ar_decode(model: OracleModel, prompt: Sequence[int], max_new: int, eos_id: i
 
 def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: int, seed: int,
                   b: int = 0, mode: str = "refill", guess_init: str = "uniform",
-                  eos_id: int = -1, record: bool = False) -> DecodeResult:
+                  eos_id: int = -1, record: bool = False, keep_steps: bool = False) -> DecodeResult:
     """Jacobi decoding with KV cache (Alg. 3) of one sequence ``b``.
 
     Each iteration forwards the current block over the committed cache,
     accepts a tokens (a >= 1), commits them (their K/V stay in the cache), and
     forms the next block from the remaining predictions (Alg. 3's
     z_next <- z_next[>= i*]); ``refill`` tops the block up to n with fresh
-    guesses, ``shrink`` lets it shrink until the window is fixed."""
+    guesses, ``shrink`` lets it shrink until the window is fixed.
+    ``record`` keeps the block of every iteration and ``keep_steps`` every
+    iteration's StepResult with its logits (recorded only, never used)."""
     assert mode in ("refill", "shrink") and n >= 1 and max_new >= 1
     V = model.arch.vocab
     src = list(prompt) if guess_init == "prompt" else None
@@ -376,7 +379,9 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
     while len(res.tokens) < max_new:
         if record:
             res.trajectory.append(list(block))
-        st = jacobi_step(sess, block, L)
+        st = jacobi_step(sess, block, L, keep_logits=keep_steps)
+        if keep_steps:
+            res.steps.append(st)
         m = len(block)
         a = st.accepted
         stop = False

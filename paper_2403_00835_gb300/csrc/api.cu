@@ -187,6 +187,7 @@ struct cllm_ctx {
   std::vector<unsigned long long> last_cta_stamps;
   int trace_phase = -1;  // profiling: phase whose MMA stage arrivals are traced
   int hold_phase = -1;   // test hook: grid barrier that cannot open (bounded-wait path)
+  bool step_logits = false;  // the step graph being built stores the LM head's logits
   std::map<std::tuple<int, int, int, int, int, unsigned long long, int, int, int, int>, GraphEntry>
       graphs;
   // profiling
@@ -677,7 +678,9 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     e.am_ticket = c->am_ticket;
     e.pred = c->pred;
     e.gap = c->gap;
-    e.logits = nullptr;
+    // single steps asked for the logits (debug/parity) store them from the
+    // same kernel that the decode loop runs
+    e.logits = (mode == MODE_STEP && c->step_logits) ? c->logits_dbg : nullptr;
     e.ssq_in = c->ssq;
     gemm_phase(EPI_ARGMAX, 7 * NL, 7 * NL, 7 * NL, mapB, ceil_div(c->V, kBM), c->V, c->d, e);
     PhaseDesc d{};
@@ -766,7 +769,7 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                              mode == MODE_DECODE ? (c->dec_opts.guess_init | (c->dec_opts.block_mode << 2) |
                                                     (c->traj_cap << 4))
                                                  : 0,
-                             c->profiling ? 1 : 0,
+                             (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0),
                              c->persistent ? 1 : 0, c->l2_ahead_persistent * 65536 + std::min(c->pre_stages, 65535));
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
@@ -1357,7 +1360,7 @@ extern "C" int cllm_jacobi_step(cllm_ctx* c, const int32_t* guess, int n, int32_
     return CLLM_ECUDA;
   if (launch_set_head(c->block, c->head, B, n, c->V, c->err, c->stream) != cudaSuccess)
     return CLLM_ECUDA;
-  if (logits_out) {
+  if (logits_out && !persistent_ok(c, B, n)) {
     std::vector<int2> qt = step_qtiles(B, n);
     if (cudaMemcpyAsync(c->qtiles_prefill, qt.data(), qt.size() * sizeof(int2),
                         cudaMemcpyHostToDevice, c->stream) != cudaSuccess)
@@ -1374,11 +1377,15 @@ extern "C" int cllm_jacobi_step(cllm_ctx* c, const int32_t* guess, int n, int32_
     f.acc = make_accept(c, B, n, false);
     if (record_forward(c, c->stream, f, false) != cudaSuccess) return CLLM_ECUDA;
   } else {
+    // the persistent kernel of the decode loop; with logits_out its LM-head
+    // phase also stores the logits
     cllm_ctx::GraphEntry* ge = nullptr;
     const bool prof = c->profiling;
     c->profiling = false;
+    c->step_logits = logits_out != nullptr;
     int rc = get_graph(c, MODE_STEP, n, &ge);
     c->profiling = prof;
+    c->step_logits = false;
     if (rc != CLLM_OK) return rc;
     cudaError_t e = cudaGraphLaunch(ge->exec, c->stream);
     if (e != cudaSuccess) return cuda_fail(e, "graph launch (step)");

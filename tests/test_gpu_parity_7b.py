@@ -10,7 +10,7 @@ torch = pytest.importorskip("torch")
 
 from oracle import oracle as orc
 from paper_2403_00835_gb300 import synthetic as syn
-from tests.parity_util import FLAG_GAP, engine_for, first_flag, logits_ok, oracle_for
+from tests.parity_util import FLAG_GAP, LOGIT_TOL_BF16, engine_for, first_flag, logits_ok, oracle_for
 
 pytestmark = pytest.mark.gpu
 
@@ -55,6 +55,46 @@ def test_7b_step_n16_prompt128(llama):
 def test_7b_step_n64_prompt512(llama):
     cfg, eng, om = llama
     _step_parity(cfg, eng, om, 512, 64)
+
+
+def test_7b_oracle_trajectory_through_persistent_kernel(llama):
+    """The oracle's own Jacobi decode (refill policy, Alg. 3 with fresh
+    guesses; prompt 128, n = 16, the benchmark's configuration) is recorded
+    block by block; each recorded block is fed to the GPU's single step, which
+    runs the persistent kernel of the decode loop.  At every iteration the
+    GPU's logits meet the bf16 bound and its predictions, gaps and accepted
+    count equal the oracle's at the rows that are not near-ties.  Inputs flow
+    from the oracle to the GPU only; the comparison stops where a near-tie
+    inside an accepted prefix could let the two states part."""
+    cfg, eng, om = llama
+    n, iters = 16, 16
+    prompt = syn.make_prompts(cfg.vocab, [128], seed=1)[0]
+    ref = orc.jacobi_decode(om, prompt, n, iters, seed=2, record=True, keep_steps=True)
+    assert ref.iterations >= iters
+    eng.prefill([prompt])
+    assert eng.uses_persistent(n)
+    L = len(prompt)
+    worst_all, flagged_all, compared = 0.0, 0, 0
+    for j, (blk, st) in enumerate(zip(ref.trajectory, ref.steps)):
+        r = eng.jacobi_step(np.asarray([blk], dtype=np.int32), want_gap=True, want_logits=True)
+        ok, worst = logits_ok(r["logits"][0], st.logits, "bf16")
+        assert ok, f"iteration {j}: logits max err / (2e-2 std) = {worst:.3f}"
+        worst_all = max(worst_all, worst)
+        for k in range(n):
+            if st.gap[k] < FLAG_GAP:
+                flagged_all += 1
+                continue
+            assert r["next"][0][k] == st.pred[k], (j, k)
+            assert abs(float(r["gap"][0][k]) - st.gap[k]) <= 2 * LOGIT_TOL_BF16 * float(np.std(st.logits[k])), (j, k)
+        compared += 1
+        if any(g < FLAG_GAP for g in st.gap[: st.accepted]):
+            break  # a near-tie inside the accepted prefix: the states may part
+        assert r["accepted"][0] == st.accepted, j
+        L += st.accepted
+        assert eng.committed_lengths()[0] == L
+    assert compared >= 8
+    print(f"{compared} iterations compared, worst logit err/bound {worst_all:.3f}, "
+          f"flagged rows {flagged_all}")
 
 
 def test_7b_decode_prefix_matches_oracle_ar(llama):

@@ -50,6 +50,29 @@ def test_persistent_steps_bit_identical(tiny_bf16, n):
     eng.set_persistent(True)
 
 
+@pytest.mark.parametrize("n", [8, 16])
+def test_persistent_logits_bit_identical(tiny_bf16, n):
+    """A step asked for its logits runs the persistent kernel (the one the
+    decode loop runs) and stores them from its LM-head phase; they equal the
+    per-GEMM path's logits bit for bit."""
+    cfg, eng = tiny_bf16
+    prompts = syn.make_prompts(cfg.vocab, [32, 17, 45], seed=1)
+    g = syn.make_guesses(cfg.vocab, 3, n, seed=2)
+    out = []
+    for persistent in (True, False):
+        eng.set_persistent(persistent)
+        eng.prefill(prompts)
+        assert eng.uses_persistent(n) == persistent
+        out.append(eng.jacobi_step(g, want_gap=True, want_logits=True))
+    eng.set_persistent(True)
+    a, b = out
+    assert np.isfinite(a["logits"]).all()
+    np.testing.assert_array_equal(a["logits"], b["logits"])
+    np.testing.assert_array_equal(a["next"], b["next"])
+    np.testing.assert_array_equal(a["gap"], b["gap"])
+    np.testing.assert_array_equal(a["accepted"], b["accepted"])
+
+
 def test_persistent_decode_bit_identical(tiny_bf16):
     cfg, eng = tiny_bf16
     prompts = syn.make_prompts(cfg.vocab, [32, 17, 45, 8], seed=5)

@@ -116,3 +116,40 @@ def test_guess_token_ranges():
     # the map from the top 32 bits is the multiply-high: r * V >> 32
     r = orc.splitmix64_output(7, orc.guess_counter(1, 2, 3) + 1) >> 32
     assert orc.guess_token(7, 1, 2, 3, V) == (r * V) >> 32
+
+
+def test_guess_token_golden_from_published_vector():
+    """Stored tokens derived from the published splitmix64 outputs: slot s of
+    sequence 0 at iteration 0 uses output s + 1."""
+    fx = json.load(open(os.path.join(GOLDEN, "guess_tokens_seed1234567.json")))
+    for V, want in fx["tokens"].items():
+        got = [orc.guess_token(fx["seed"], fx["b"], fx["step"], s, int(V)) for s in fx["slots"]]
+        assert got == want, V
+    picks = [orc.guess_token(fx["seed"], 0, 0, s, 32000, fx["prompt"]) for s in fx["slots"]]
+    assert picks == fx["prompt_picks"]
+
+
+def _splitmix64_sequential(seed, count):
+    """The generator as published: a 64-bit state advanced by the golden-ratio
+    increment before each output, then the three-step mix.  Yields `count`
+    outputs in order."""
+    m = (1 << 64) - 1
+    state = seed & m
+    for _ in range(count):
+        state = (state + 0x9E3779B97F4A7C15) & m
+        z = state
+        z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & m
+        z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & m
+        yield z ^ (z >> 31)
+
+
+def test_guess_token_counter_layout_by_sequential_generator():
+    """The counter-based draw for (iteration j, slot s) of sequence 0 is the
+    (j * 2^16 + s + 1)-th output of the sequential generator."""
+    V, seed = 32000, 1234567
+    outs = list(_splitmix64_sequential(seed, (1 << 16) + 8))
+    fx = json.load(open(os.path.join(GOLDEN, "splitmix64_seed1234567.json")))
+    assert outs[:5] == [int(s) for s in fx["outputs"]]
+    for step, slot in ((0, 0), (0, 7), (1, 0), (1, 3)):
+        i = (step << 16) + slot  # 0-based index of the output
+        assert orc.guess_token(seed, 0, step, slot, V) == ((outs[i] >> 32) * V) >> 32, (step, slot)
