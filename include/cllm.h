@@ -272,11 +272,14 @@ int cllm_committed_lengths(cllm_ctx *ctx, int32_t *lens_out);
  * No memory is allocated: all scratch (split-K partial tiles, arrival tickets,
  * the device error word, epilogue side outputs) lives in one static device
  * array of 8 MiB that each device loading the library holds until exit.  Sizes
- * whose scratch would exceed it return CLLM_ECAPACITY before any launch.  The
- * first call on a device looks up that array's device address; make it before
- * any stream capture.  Every call reuses the same array (tickets and the error
- * word are cleared at the start of each call), so calls that overlap on the
- * GPU -- from several threads or streams -- race and must not be issued.
+ * whose scratch would exceed it return CLLM_ECAPACITY before any launch.  Each
+ * call looks up the array's device address in the current device's current
+ * context (a host-side lookup), so a reset device or a second context on the
+ * same device gets its own copy.  Every call reuses the same array (tickets
+ * and the error word are cleared at the start of each call; the rest keeps
+ * the previous call's contents and is overwritten before it is read), so calls
+ * that overlap on the GPU -- from several threads or streams -- race and must
+ * not be issued.
  * Returns CLLM_OK, EINVAL, ECAPACITY, EUNSUPPORTED, ECUDA, EDEVICE or ETIMEOUT.
  */
 int cllm_gemm_bf16_noalloc(const void *W, const void *X, float *Y, int M, int K, int T,

@@ -22,10 +22,6 @@
 
 using namespace cllm;
 
-// Weight tiles per CTA prefetched into L2 ahead of the shared-memory ring.
-// Measured on chains of GEMM launches: it adds traffic without shortening the
-// chain, so it is off.
-static constexpr int kL2AheadDefault = 0;
 
 namespace cllm {
 

@@ -24,6 +24,10 @@ constexpr int kQTile = 16;       // query rows per attention tile
 constexpr int kBK = 64;          // K elements per pipeline stage (128 B of bf16)
 constexpr int kBM = 128;         // weight rows per tile (MMA M)
 constexpr int kEpiCols = 16;     // columns per epilogue chunk
+// Weight tiles per CTA prefetched into L2 ahead of the shared-memory ring by
+// the per-GEMM kernels.  Measured on chains of GEMM launches: it adds traffic
+// without shortening the chain, so it is off.
+constexpr int kL2AheadDefault = 0;
 
 enum EpiKind : int { EPI_QKV = 0, EPI_GATEUP = 1, EPI_RESID = 2, EPI_ARGMAX = 3 };
 

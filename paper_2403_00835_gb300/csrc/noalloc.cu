@@ -8,8 +8,6 @@
 // partial tiles, arrival tickets, the device error word, and the epilogue's
 // side outputs) lives in one file-scope device array of fixed size, so the
 // call allocates nothing.  The caller still provides the inputs and output.
-#include <mutex>
-
 #include "../../include/cllm.h"
 #include "internal.cuh"
 
@@ -23,23 +21,16 @@ constexpr size_t kNoAllocScratchBytes = size_t(8) << 20;  // 8 MiB, held by each
 // only a stand-in: its device address comes from cudaGetSymbolAddress.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-void* g_scratch_addr[kMaxDevices] = {};
-
-// Device address of the scratch array on the current device, looked up once
-// per device (the first call on a device does this set-up).
+// Device address of the scratch array in the current device's current
+// context.  It is looked up on every call (a host-side table lookup, cheap):
+// an address cached per device would be stale after cudaDeviceReset or in a
+// second driver context on the same device, and the kernel would then write
+// its partial sums into memory it does not own.  The first call in a context
+// also loads the library's device code there.
 int scratch_address(void** out) {
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return CLLM_ECUDA;
-  if (dev < 0 || dev >= kMaxDevices) return CLLM_EUNSUPPORTED;
-  std::lock_guard<std::mutex> lk(g_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return CLLM_ECUDA;
-    g_scratch_addr[dev] = p;
-  }
-  *out = g_scratch_addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return CLLM_ECUDA;
+  *out = p;
   return CLLM_OK;
 }
 
@@ -112,7 +103,7 @@ extern "C" int cllm_gemm_bf16_noalloc(const void* W, const void* X, float* Y, in
   g.rows_q = M;
   g.rows_qk = M;
   g.lo_rows = x_rows;
-  g.l2_ahead = 16;
+  g.l2_ahead = kL2AheadDefault;  // as the allocating GEMM entry points
   g.pre_stages = 1 << 20;
   g.partial = reinterpret_cast<float*>(sb + off_part);
   g.tickets = reinterpret_cast<int*>(sb + off_tick);

@@ -37,22 +37,34 @@ def _inputs(M, K, T, seed):
 
 @pytest.mark.parametrize("M,K,T", [(4096, 4096, 16), (768, 688, 17)])
 def test_noalloc_matches_allocating_gemm_twice(M, K, T):
+    """Y is accumulated into: both entry points start from the same nonzero Y0
+    and must give Y0 + W.X.  The second call must not change the device's
+    free memory or the caching allocator's reservation."""
     lib = _lib()
     stream = torch.cuda.current_stream()
     for call in range(2):
         W, X2, rows = _inputs(M, K, T, seed=100 * call + M + K + T)
-        ref = torch.zeros(T, M, device="cuda", dtype=torch.float32)
+        g = torch.Generator(device="cuda").manual_seed(7 + call)
+        Y0 = torch.randn(T, M, device="cuda", generator=g)
+        ref = Y0.clone()
         assert lib.cllm_test_gemm_bf16(W.data_ptr(), X2.data_ptr(), ref.data_ptr(), M, K, T, rows) == 0
-        out = torch.zeros(T, M, device="cuda", dtype=torch.float32)
+        out = Y0.clone()
+        torch.cuda.synchronize()
+        free0, reserved0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_reserved()
         rc = lib.cllm_gemm_bf16_noalloc(W.data_ptr(), X2.data_ptr(), out.data_ptr(), M, K, T, rows,
                                         ctypes.c_void_p(stream.cuda_stream))
         assert rc == 0, cllm.STATUS.get(rc, rc)
         torch.cuda.synchronize()
+        if call == 1:  # the first call may load the library's device code
+            assert torch.cuda.mem_get_info()[0] == free0
+            assert torch.cuda.memory_reserved() == reserved0
         Wd = W.cpu().double().numpy()
         Xd = (X2[0, :T].double() + X2[1, :T].double()).cpu().numpy()
-        bound = 1e-5 * (np.abs(Xd) @ np.abs(Wd).T) + 1e-7
+        exact = Y0.cpu().double().numpy() + Xd @ Wd.T
+        bound = 1e-5 * (np.abs(Xd) @ np.abs(Wd).T + np.abs(Y0.cpu().double().numpy())) + 1e-7
         diff = np.abs(out.cpu().double().numpy() - ref.cpu().double().numpy())
         assert (diff <= bound).all(), float((diff / bound).max())
+        assert (np.abs(out.cpu().double().numpy() - exact) <= 4e-3 * np.abs(exact).max()).all()
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch():
