@@ -96,7 +96,18 @@ typedef struct {
   int block_mode;  /* CLLM_BLOCK_REFILL | CLLM_BLOCK_SHRINK                       */
   int record_cap;  /* > 0: record the first record_cap blocks of every sequence
                       (the Jacobi trajectory), read with cllm_decode_read_trajectory */
+  int stats;       /* 1: keep the acceptance statistics on the device, read with
+                      cllm_decode_read_stats; 0: off                           */
 } cllm_decode_opts;
+
+/* Acceptance statistics of a decode (Sec. 3.3, Table 3), summed over the
+ * batch.  See cllm_decode_read_stats. */
+typedef struct {
+  int64_t iterations; /* sequence-iterations run                                  */
+  int64_t accepted;   /* tokens they committed (fast-forwarded, head included)     */
+  int64_t windows;    /* n-token windows opened                                   */
+  int64_t stationary; /* stationary tokens inside those windows                   */
+} cllm_accept_stats;
 
 typedef struct cllm_ctx cllm_ctx;
 
@@ -212,6 +223,29 @@ int cllm_decode_read(cllm_ctx *ctx, int32_t *tokens_out, int32_t *iters_out);
  * did not run are -1.  Host buffer of record_cap*B*n ints, owned by the
  * caller.  ESTATE when the decode did not record. */
 int cllm_decode_read_trajectory(cllm_ctx *ctx, int32_t *blocks_out);
+
+/*
+ * Acceptance statistics of the decode in progress (or just finished), kept
+ * on the device by the accept step when cllm_decode_begin's opts->stats = 1
+ * (Sec. 3.3 and Table 3 define both quantities in words):
+ *  - fast-forwarded count of an iteration: its accepted count a (the head
+ *    included, as Table 3 counts it).  acc_hist[a] (host, [n+1] or NULL) =
+ *    sequence-iterations that accepted a tokens; out->iterations and
+ *    out->accepted are its count and weighted sum.
+ *  - stationary tokens: a position is stationary when, before it is
+ *    committed, it already holds its final token while an earlier slot of the
+ *    block is wrong, and keeps it in every later block until it is committed.
+ *    A window is the run of positions covered by the first block that starts
+ *    at or after the previous window's end (under CLLM_BLOCK_SHRINK exactly
+ *    one n-token window of Alg. 3); stationary tokens count toward the window
+ *    that holds them.  win_hist[s] (host, [n+1] or NULL) = windows with s
+ *    stationary tokens, windows still open included; out->windows and
+ *    out->stationary are the totals.
+ * Synchronises the context's stream.  ESTATE without a decode begun with
+ * stats = 1; EINVAL on a null ctx or out.
+ */
+int cllm_decode_read_stats(cllm_ctx *ctx, cllm_accept_stats *out, int64_t *acc_hist,
+                           int64_t *win_hist);
 
 /* ---- options --------------------------------------------------------------------
  * CLLM_OPT_PERSISTENT (default 1): run each decode/step iteration of the bf16

@@ -29,7 +29,7 @@ EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "c
            "cllm_decode_read", "cllm_set_profiling", "cllm_profile_read",
            "cllm_kernels_per_iteration", "cllm_committed_lengths", "cllm_gemm_bf16_noalloc",
            "cllm_set_option", "cllm_uses_persistent", "cllm_last_cuda_error",
-           "cllm_decode_read_trajectory")
+           "cllm_decode_read_trajectory", "cllm_decode_read_stats")
 CLLM_OPT_PERSISTENT = 1
 CLLM_OPT_L2_AHEAD = 2
 CLLM_OPT_PRE_STAGES = 3
@@ -61,7 +61,12 @@ class Weights(ctypes.Structure):
 
 class DecodeOpts(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("eos_id", ctypes.c_int), ("guess_init", ctypes.c_int),
-                ("block_mode", ctypes.c_int), ("record_cap", ctypes.c_int)]
+                ("block_mode", ctypes.c_int), ("record_cap", ctypes.c_int), ("stats", ctypes.c_int)]
+
+
+class AcceptStats(ctypes.Structure):
+    _fields_ = [("iterations", ctypes.c_int64), ("accepted", ctypes.c_int64),
+                ("windows", ctypes.c_int64), ("stationary", ctypes.c_int64)]
 
 
 _lib = None
@@ -113,6 +118,9 @@ def load(build_if_missing: bool = True):
     lib.cllm_uses_persistent.argtypes = [vp, ctypes.c_int]
     lib.cllm_uses_persistent.restype = ctypes.c_int
     lib.cllm_decode_read_trajectory.argtypes = [vp, i32p]
+    i64p = ctypes.POINTER(ctypes.c_int64)
+    lib.cllm_decode_read_stats.argtypes = [vp, ctypes.POINTER(AcceptStats), i64p, i64p]
+    lib.cllm_decode_read_stats.restype = ctypes.c_int
     lib.cllm_last_cuda_error.argtypes = []
     lib.cllm_last_cuda_error.restype = ctypes.c_char_p
     for name in ("cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode", "cllm_ar_decode",
@@ -229,21 +237,23 @@ class Engine:
 
     def jacobi_decode(self, prompts, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
                       guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL,
-                      record_cap: int = 0):
+                      record_cap: int = 0, stats: bool = False):
         """Tokens [B][max_new] and iterations [B]; with record_cap > 0 also the
-        trajectory [record_cap][B][n] (-1 outside the window)."""
+        trajectory [record_cap][B][n] (-1 outside the window).  With stats the
+        device keeps the acceptance statistics (read with decode_read_stats)."""
         toks, lens = _flatten_prompts(prompts)
         B = len(prompts)
         out = np.zeros((B, max_new), dtype=np.int32)
         its = np.zeros(B, dtype=np.int32)
-        o = DecodeOpts(seed, eos_id, guess_init, block_mode, record_cap)
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, record_cap, 1 if stats else 0)
         _check(self._lib.cllm_jacobi_decode(self._h, B, _ip(toks), _ip(lens), n, max_new,
                                             ctypes.byref(o), _ip(out), _ip(its)), "cllm_jacobi_decode")
         self.B = B
+        self._dec_n = n
         if record_cap > 0:
             traj = np.zeros((record_cap, B, n), dtype=np.int32)
             _check(self._lib.cllm_decode_read_trajectory(self._h, _ip(traj)),
-                   "cllm_decode_read_trajectory")
+                   "cllm_decode_read_trajectory", "cllm_decode_read_stats")
             return out, its, traj
         return out, its
 
@@ -257,10 +267,28 @@ class Engine:
         return out
 
     def decode_begin(self, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
-                     guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL):
-        o = DecodeOpts(seed, eos_id, guess_init, block_mode, 0)
+                     guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL,
+                     stats: bool = False):
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, 0, 1 if stats else 0)
         _check(self._lib.cllm_decode_begin(self._h, n, max_new, ctypes.byref(o)), "cllm_decode_begin")
         self._dec_max_new = max_new
+        self._dec_n = n
+
+    def decode_read_stats(self):
+        """The device's acceptance statistics of the current decode: totals
+        (iterations, accepted, windows, stationary) and the histograms
+        acc_hist[a] (iterations accepting a tokens) and win_hist[s] (windows
+        with s stationary tokens), both [n + 1]."""
+        n = self._dec_n
+        st = AcceptStats()
+        ah = np.zeros(n + 1, dtype=np.int64)
+        wh = np.zeros(n + 1, dtype=np.int64)
+        _check(self._lib.cllm_decode_read_stats(self._h, ctypes.byref(st),
+                                                ah.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
+                                                wh.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))),
+               "cllm_decode_read_stats")
+        return {"iterations": st.iterations, "accepted": st.accepted, "windows": st.windows,
+                "stationary": st.stationary, "acc_hist": ah, "win_hist": wh}
 
     def decode_run(self, max_iters: int):
         it = ctypes.c_int(0)

@@ -150,6 +150,11 @@ struct cllm_ctx {
       *iters = nullptr, *done = nullptr, *out = nullptr, *accepted = nullptr, *prompts = nullptr,
       *plen = nullptr, *status = nullptr, *err = nullptr, *width = nullptr;
   size_t out_cap = 0;
+  // acceptance statistics (cllm_decode_opts.stats): histograms [max_block+1],
+  // totals [2], per-sequence slot state [max_batch][max_block], windows [max_batch]
+  unsigned long long *acc_hist = nullptr, *win_hist = nullptr, *st_totals = nullptr;
+  int *st_pos = nullptr, *st_val = nullptr, *st_cand = nullptr, *win_end = nullptr,
+      *win_cnt = nullptr;
   int* traj = nullptr;  // recorded trajectory [traj_cap][B][n]
   size_t traj_alloc = 0;
   int traj_cap = 0;
@@ -535,6 +540,16 @@ AcceptArgs make_accept(cllm_ctx* c, int B, int n, bool decode) {
   a.width = c->width;
   a.traj = (decode && c->traj_cap > 0) ? c->traj : nullptr;
   a.traj_cap = decode ? c->traj_cap : 0;
+  if (decode && c->dec_opts.stats) {
+    a.acc_hist = c->acc_hist;
+    a.win_hist = c->win_hist;
+    a.totals = c->st_totals;
+    a.st_pos = c->st_pos;
+    a.st_val = c->st_val;
+    a.st_cand = c->st_cand;
+    a.win_end = c->win_end;
+    a.win_cnt = c->win_cnt;
+  }
   return a;
 }
 
@@ -765,7 +780,8 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                              mode == MODE_DECODE ? (c->dec_opts.guess_init | (c->dec_opts.block_mode << 2) |
                                                     (c->traj_cap << 4))
                                                  : 0,
-                             (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0),
+                             (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0) |
+                                 (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0),
                              c->persistent ? 1 : 0, c->l2_ahead_persistent * 65536 + std::min(c->pre_stages, 65535));
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
@@ -1193,6 +1209,12 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
          dev_alloc(c, &c->committed, Bm * 4) && dev_alloc(c, &c->iters, Bm * 4) &&
          dev_alloc(c, &c->done, Bm * 4) && dev_alloc(c, &c->accepted, Bm * 4) &&
          dev_alloc(c, &c->width, Bm * 4) &&
+         dev_alloc(c, &c->acc_hist, (a.max_block + 1) * 8) &&
+         dev_alloc(c, &c->win_hist, (a.max_block + 1) * 8) && dev_alloc(c, &c->st_totals, 16) &&
+         dev_alloc(c, &c->st_pos, Bm * a.max_block * 4) &&
+         dev_alloc(c, &c->st_val, Bm * a.max_block * 4) &&
+         dev_alloc(c, &c->st_cand, Bm * a.max_block * 4) && dev_alloc(c, &c->win_end, Bm * 4) &&
+         dev_alloc(c, &c->win_cnt, Bm * 4) &&
          dev_alloc(c, &c->prompts, Bm * a.max_seq * 4) && dev_alloc(c, &c->plen, Bm * 4) &&
          dev_alloc(c, &c->status, 16) && dev_alloc(c, &c->err, 16);
     if (!ok) {
@@ -1419,6 +1441,7 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
   if (o.guess_init != CLLM_GUESS_UNIFORM && o.guess_init != CLLM_GUESS_FROM_PROMPT) return CLLM_EINVAL;
   if (o.block_mode != CLLM_BLOCK_REFILL && o.block_mode != CLLM_BLOCK_SHRINK) return CLLM_EINVAL;
   if (o.record_cap < 0 || o.record_cap > (1 << 20)) return CLLM_EINVAL;
+  if (o.stats != 0 && o.stats != 1) return CLLM_EINVAL;
   if (o.eos_id >= c->V) return CLLM_EINVAL;
   for (int b = 0; b < c->B; ++b)
     if (static_cast<long>(c->lens[b]) + max_new + n > c->arch.max_seq) return CLLM_ECAPACITY;
@@ -1551,6 +1574,40 @@ extern "C" int cllm_decode_read_trajectory(cllm_ctx* c, int32_t* blocks_out) {
   if (cudaMemcpyAsync(blocks_out, c->traj, bytes, cudaMemcpyDeviceToHost, c->stream) != cudaSuccess)
     return cuda_fail(cudaGetLastError(), "trajectory copy");
   return check_device_error(c);
+}
+
+extern "C" int cllm_decode_read_stats(cllm_ctx* c, cllm_accept_stats* out, int64_t* acc_hist,
+                                     int64_t* win_hist) {
+  if (!c || !out) return CLLM_EINVAL;
+  if (!c->dec_active || !c->dec_opts.stats) return CLLM_ESTATE;
+  cudaSetDevice(c->dev);
+  const int n = c->dec_n, B = c->B;
+  std::vector<unsigned long long> ah(n + 1), wh(n + 1), tot(2);
+  std::vector<int> wend(B), wcnt(B);
+  if (cudaMemcpyAsync(ah.data(), c->acc_hist, (n + 1) * 8, cudaMemcpyDeviceToHost, c->stream) ||
+      cudaMemcpyAsync(wh.data(), c->win_hist, (n + 1) * 8, cudaMemcpyDeviceToHost, c->stream) ||
+      cudaMemcpyAsync(tot.data(), c->st_totals, 16, cudaMemcpyDeviceToHost, c->stream) ||
+      cudaMemcpyAsync(wend.data(), c->win_end, B * 4, cudaMemcpyDeviceToHost, c->stream) ||
+      cudaMemcpyAsync(wcnt.data(), c->win_cnt, B * 4, cudaMemcpyDeviceToHost, c->stream))
+    return cuda_fail(cudaGetLastError(), "statistics copy");
+  const int rc = check_device_error(c);  // synchronises
+  if (rc != CLLM_OK) return rc;
+  // windows still open count with their stationary tokens so far
+  for (int b = 0; b < B; ++b)
+    if (wend[b] > 0) wh[std::min(wcnt[b], n)] += 1;
+  cllm_accept_stats st{};
+  for (int a = 0; a <= n; ++a) {
+    st.iterations += static_cast<int64_t>(ah[a]);
+    st.accepted += static_cast<int64_t>(ah[a]) * a;
+  }
+  st.windows = static_cast<int64_t>(tot[0]);
+  st.stationary = static_cast<int64_t>(tot[1]);
+  *out = st;
+  for (int a = 0; a <= n; ++a) {
+    if (acc_hist) acc_hist[a] = static_cast<int64_t>(ah[a]);
+    if (win_hist) win_hist[a] = static_cast<int64_t>(wh[a]);
+  }
+  return CLLM_OK;
 }
 
 extern "C" int cllm_jacobi_decode(cllm_ctx* c, int B, const int32_t* tokens, const int32_t* lens,

@@ -169,6 +169,22 @@ struct AcceptArgs {
   // iteration it (slot k < width, -1 beyond), for it < traj_cap
   int* traj;
   int traj_cap;
+  // acceptance statistics of a decode (Sec. 3.3, Table 3), kept on the device
+  // (null: off).  acc_hist[a]: sequence-iterations that accepted a tokens;
+  // win_hist[s]: closed n-token windows with s stationary tokens; totals[0]
+  // windows opened, totals[1] stationary tokens inside windows.  Per sequence
+  // b and window slot q = position mod n: st_pos/st_val the position and value
+  // the slot last held, st_cand whether, since that value arrived, an earlier
+  // slot of the block was wrong; win_end/win_cnt the open window's end and its
+  // stationary count.  Positions count committed tokens from the decode start.
+  unsigned long long* acc_hist;  // [n + 1]
+  unsigned long long* win_hist;  // [n + 1]
+  unsigned long long* totals;    // [2]
+  int* st_pos;                   // [B][n]
+  int* st_val;                   // [B][n]
+  int* st_cand;                  // [B][n]
+  int* win_end;                  // [B]
+  int* win_cnt;                  // [B]
 };
 
 // ---- persistent per-iteration kernel (persistent.cu) ---------------------------------

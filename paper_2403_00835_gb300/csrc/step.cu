@@ -45,6 +45,18 @@ __global__ void __launch_bounds__(128) decode_init_kernel(const AcceptArgs a) {
     int* y = a.block + b * a.n;
     y[0] = a.head[b];
     for (int k = 1; k < a.n; ++k) y[k] = draw_guess(a, b, 0, k);
+    if (a.acc_hist != nullptr) {
+      a.win_end[b] = 0;
+      a.win_cnt[b] = 0;
+      for (int k = 0; k < a.n; ++k) a.st_pos[static_cast<size_t>(b) * a.n + k] = -1;
+    }
+  }
+  if (a.acc_hist != nullptr) {
+    for (int i = tid; i <= a.n; i += blockDim.x) {
+      a.acc_hist[i] = 0;
+      a.win_hist[i] = 0;
+    }
+    if (tid < 2) a.totals[tid] = 0;
   }
   for (size_t i = tid; i < static_cast<size_t>(a.B) * a.max_new; i += blockDim.x) a.out[i] = -1;
   if (tid == 0) {

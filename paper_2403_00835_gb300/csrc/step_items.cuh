@@ -71,6 +71,55 @@ __device__ void embed_unit(const EmbedArgs& a, int t, int grp, int i, float* red
   sync();  // red[] is reused by the next unit
 }
 
+// Acceptance statistics of one iteration of sequence b (decode loop): the
+// block y of active width w commits acc tokens at positions c..c+acc-1,
+// c = tokens committed so far.  Fast-forwarded count (Table 3): acc itself,
+// the head included.  Stationary tokens (Sec. 3.3): a position is
+// stationary when, before it is committed, it already holds its final token
+// while an earlier slot of the block is wrong, and keeps that token in every
+// later block until it is committed.  Kept online: a slot's candidate flag
+// is set when it holds an unchanged value at an iteration whose accepted
+// prefix ends before it, and restarts whenever its value changes; a committed
+// token is final, so a committed position is stationary exactly when its flag
+// is set.  Windows: a window opens with the first block that starts at or
+// after the previous window's end and covers that block's w positions;
+// stationary positions count toward the window that holds them.
+__device__ inline void accept_stats(const AcceptArgs& a, int b, const int* y, int w, int acc) {
+  const int n = a.n;
+  const int c = a.committed[b];
+  int* pos = a.st_pos + static_cast<size_t>(b) * n;
+  int* val = a.st_val + static_cast<size_t>(b) * n;
+  int* cand = a.st_cand + static_cast<size_t>(b) * n;
+  if (c >= a.win_end[b]) {
+    if (a.win_end[b] > 0) atomicAdd(&a.win_hist[min(a.win_cnt[b], n)], 1ull);
+    a.win_end[b] = c + w;
+    a.win_cnt[b] = 0;
+    atomicAdd(&a.totals[0], 1ull);
+  }
+  atomicAdd(&a.acc_hist[min(acc, n)], 1ull);
+  for (int k = 0; k < w; ++k) {
+    const int p = c + k, q = p % n;
+    const int later = k > acc ? 1 : 0;
+    if (pos[q] != p || val[q] != y[k]) {
+      pos[q] = p;
+      val[q] = y[k];
+      cand[q] = later;
+    } else {
+      cand[q] |= later;
+    }
+  }
+  int found = 0;
+  for (int k = 0; k < acc; ++k) {
+    const int p = c + k, q = p % n;
+    if (cand[q] && p < a.win_end[b]) ++found;
+    pos[q] = -1;  // committed: the slot's next position starts afresh
+  }
+  if (found) {
+    a.win_cnt[b] += found;
+    atomicAdd(&a.totals[1], static_cast<unsigned long long>(found));
+  }
+}
+
 template <class Sync>
 __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, Sync sync) {
   int active = 0, committed_now = 0;
@@ -98,6 +147,7 @@ __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, 
         }
         const int room = a.max_new - a.committed[b];
         if (acc > room) acc = room;
+        if (a.acc_hist != nullptr) accept_stats(a, b, y, w, acc);
         int* out = a.out + static_cast<size_t>(b) * a.max_new + a.committed[b];
         for (int k = 0; k < acc; ++k) out[k] = y[k];
         a.committed[b] += acc;

@@ -64,17 +64,19 @@ def test_7b_oracle_trajectory_through_persistent_kernel(llama):
     runs the persistent kernel of the decode loop.  At every iteration the
     GPU's logits meet the bf16 bound and its predictions, gaps and accepted
     count equal the oracle's at the rows that are not near-ties.  Inputs flow
-    from the oracle to the GPU only; the comparison stops where a near-tie
-    inside an accepted prefix could let the two states part."""
+    from the oracle to the GPU only.  A near-tie inside the accepted prefix
+    may let the GPU commit differently; the comparison goes on while the GPU's
+    accepted count and next head still equal the oracle's (the two states are
+    then identical) and stops at the first actual parting."""
     cfg, eng, om = llama
-    n, iters = 16, 16
+    n, iters = 16, 20
     prompt = syn.make_prompts(cfg.vocab, [128], seed=1)[0]
     ref = orc.jacobi_decode(om, prompt, n, iters, seed=2, record=True, keep_steps=True)
-    assert ref.iterations >= iters
+    assert ref.iterations >= 16
     eng.prefill([prompt])
     assert eng.uses_persistent(n)
     L = len(prompt)
-    worst_all, flagged_all, compared = 0.0, 0, 0
+    worst_all, flagged_all, compared, parted = 0.0, 0, 0, None
     for j, (blk, st) in enumerate(zip(ref.trajectory, ref.steps)):
         r = eng.jacobi_step(np.asarray([blk], dtype=np.int32), want_gap=True, want_logits=True)
         ok, worst = logits_ok(r["logits"][0], st.logits, "bf16")
@@ -87,14 +89,17 @@ def test_7b_oracle_trajectory_through_persistent_kernel(llama):
             assert r["next"][0][k] == st.pred[k], (j, k)
             assert abs(float(r["gap"][0][k]) - st.gap[k]) <= 2 * LOGIT_TOL_BF16 * float(np.std(st.logits[k])), (j, k)
         compared += 1
-        if any(g < FLAG_GAP for g in st.gap[: st.accepted]):
-            break  # a near-tie inside the accepted prefix: the states may part
-        assert r["accepted"][0] == st.accepted, j
-        L += st.accepted
+        a = st.accepted
+        same = r["accepted"][0] == a and r["next"][0][a - 1] == st.pred[a - 1]
+        if any(g < FLAG_GAP for g in st.gap[:a]) and not same:
+            parted = j  # decided by a near-tie: the two states part here
+            break
+        assert same, j
+        L += a
         assert eng.committed_lengths()[0] == L
-    assert compared >= 8
-    print(f"{compared} iterations compared, worst logit err/bound {worst_all:.3f}, "
-          f"flagged rows {flagged_all}")
+    assert compared >= 16 or (parted is not None and compared >= 4), (compared, parted)
+    print(f"{compared} iterations compared (parted at {parted}), worst logit err/bound "
+          f"{worst_all:.3f}, flagged rows {flagged_all}")
 
 
 def test_7b_decode_prefix_matches_oracle_ar(llama):
