@@ -256,15 +256,13 @@ int cllm_decode_read_stats(cllm_ctx *ctx, cllm_accept_stats *out, int64_t *acc_h
  * captured after the call.  Returns CLLM_OK or EINVAL (unknown option).
  */
 #define CLLM_OPT_PERSISTENT 1
-/* CLLM_OPT_PRE_STAGES (default: the whole ring): in the persistent kernel,
- * weight tiles per CTA issued for the next GEMM phase before its grid barrier
- * opens. */
-#define CLLM_OPT_PRE_STAGES 3
-/* CLLM_OPT_L2_AHEAD (default 0): in the persistent kernel, weight tiles
- * (16 KB each) per CTA that the TMA producer prefetches into L2 for the next
- * GEMM phase once its shared-memory ring is full, while the previous phase
- * drains.  0..4096. */
-#define CLLM_OPT_L2_AHEAD 2
+/* CLLM_OPT_PARK_SLOTS (default 0 = all): in the persistent kernel, the weight
+ * tiles (16 KB each) a CTA may hold in tensor memory ahead of its MMAs.  The
+ * weight stream runs ahead of the grid barriers into these slots, so HBM keeps
+ * streaming while a phase drains; 1..64 limits it (values above the kernel's
+ * slot count mean all).  Results do not depend on it.  Takes effect for
+ * graphs captured after the call. */
+#define CLLM_OPT_PARK_SLOTS 3
 int cllm_set_option(cllm_ctx *ctx, int option, int value);
 
 /* 1 if an iteration of width n on the current batch runs as the persistent

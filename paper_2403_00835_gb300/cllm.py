@@ -31,8 +31,7 @@ EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "c
            "cllm_set_option", "cllm_uses_persistent", "cllm_last_cuda_error",
            "cllm_decode_read_trajectory", "cllm_decode_read_stats")
 CLLM_OPT_PERSISTENT = 1
-CLLM_OPT_L2_AHEAD = 2
-CLLM_OPT_PRE_STAGES = 3
+CLLM_OPT_PARK_SLOTS = 3
 
 
 class CllmError(RuntimeError):
@@ -306,11 +305,8 @@ class Engine:
     def set_persistent(self, on: bool):
         _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PERSISTENT, 1 if on else 0), "cllm_set_option")
 
-    def set_l2_ahead(self, tiles: int):
-        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_L2_AHEAD, int(tiles)), "cllm_set_option")
-
-    def set_pre_stages(self, tiles: int):
-        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PRE_STAGES, int(tiles)), "cllm_set_option")
+    def set_park_slots(self, tiles: int):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PARK_SLOTS, int(tiles)), "cllm_set_option")
 
     def uses_persistent(self, n: int) -> bool:
         r = self._lib.cllm_uses_persistent(self._h, n)

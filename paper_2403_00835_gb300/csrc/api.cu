@@ -60,17 +60,22 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, 
 // Split of one GEMM launch over the SMs.  T <= 256: one N-tile holding every
 // token and the (tile, k-chunk) space cut into equal contiguous ranges; the
 // cut depends on the weight shape and the SM count only.  T > 256: whole
-// 128 x 256 tiles per CTA, no split.
+// 128 x 256 tiles per CTA, no split.  Chunks per tile and per CTA are even,
+// so that every range and every tile starts on a pair of chunks: the
+// persistent kernel moves weights in pairs (32 KB per pipeline stage), in the
+// same order as the per-chunk kernels, which keeps the two paths bit-identical.
+// (A K that is not a multiple of 128 gets one chunk past its end, which TMA
+// fills with zeros.)
 Part plan_gemm(int mtiles, int K, int T, int sms) {
   Part p{};
   p.mtiles = mtiles;
-  p.kchunks = ceil_div(K, kBK);
+  p.kchunks = round_up(ceil_div(K, kBK), 2);
   if (T <= 256) {
     p.ntiles = 1;
     p.bn = round_up(std::max(T, 1), 16);
     p.bn_max = p.bn <= 32 ? 32 : (p.bn <= 64 ? 64 : (p.bn <= 128 ? 128 : 256));
     const int C = mtiles * p.kchunks;
-    p.cpc = ceil_div(C, sms);
+    p.cpc = round_up(ceil_div(C, sms), 2);
     p.grid = ceil_div(C, p.cpc);
     p.maxc = 1;
     for (int u = 0; u < mtiles; ++u) {
@@ -181,8 +186,7 @@ struct cllm_ctx {
     unsigned long long* cta_stamps = nullptr;
   };
   bool persistent = true;  // one persistent kernel per iteration where supported
-  int l2_ahead_persistent = 0;  // weight tiles per CTA prefetched into L2 at a barrier
-  int pre_stages = 1 << 20;     // weight tiles issued before a phase's barrier opens
+  int park_slots = 0;  // persistent kernel: tensor-memory park slots in use (0: all)
   std::vector<unsigned long long> last_stamps;  // last profiled persistent iteration
   std::vector<std::string> last_phase_names;
   std::vector<unsigned long long> last_cta_stamps;
@@ -637,10 +641,9 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     d.map_b = mb;
     Part p;
     d.g = tc_gemm_args(c, mtiles, M, K, T, e, &p);
-    d.g.l2_ahead = c->l2_ahead_persistent;
-    d.g.pre_stages = c->pre_stages;
     d.e = e;
-    bn_max = p.bn_max;
+    // the persistent kernel also has a 16-column variant (4 KB activation tiles)
+    bn_max = p.bn <= 16 ? 16 : p.bn_max;
     ph.push_back(d);
   };
   {
@@ -760,6 +763,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   sa.map_attn_k = mapA;
   sa.map_attn_v = mapA + 1;
   sa.map_attn_q = mapA + 2;
+  sa.park_limit = c->park_slots;
   sa.err = c->err;
   return CLLM_OK;
 }
@@ -782,7 +786,7 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                                                  : 0,
                              (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0) |
                                  (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0),
-                             c->persistent ? 1 : 0, c->l2_ahead_persistent * 65536 + std::min(c->pre_stages, 65535));
+                             c->persistent ? 1 : 0, c->park_slots);
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
     *out = &it->second;
@@ -1645,14 +1649,9 @@ extern "C" int cllm_set_option(cllm_ctx* c, int option, int value) {
     c->persistent = value != 0;
     return CLLM_OK;
   }
-  if (option == CLLM_OPT_PRE_STAGES) {
-    if (value < 0) return CLLM_EINVAL;
-    c->pre_stages = value;
-    return CLLM_OK;
-  }
-  if (option == CLLM_OPT_L2_AHEAD) {
-    if (value < 0 || value > 4096) return CLLM_EINVAL;
-    c->l2_ahead_persistent = value;
+  if (option == CLLM_OPT_PARK_SLOTS) {
+    if (value < -1 || value > 64) return CLLM_EINVAL;
+    c->park_slots = value;
     return CLLM_OK;
   }
   return CLLM_EINVAL;

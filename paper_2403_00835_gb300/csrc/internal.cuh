@@ -223,6 +223,9 @@ struct StepArgs {
   int hold_phase;
   // attention tile loads: indices of the K-cache, V-cache and Q tensor maps
   int map_attn_k, map_attn_v, map_attn_q;
+  // tensor-memory park slots the weight stream may fill ahead of the MMAs
+  // (0: all the kernel has)
+  int park_limit;
   int* err;
 };
 
@@ -241,7 +244,7 @@ struct StepParams {
 };
 static_assert(sizeof(StepParams) <= 32764, "kernel parameter space");
 
-// Launch of the persistent kernel (bn_max 32/64/128, head_dim 64/128).
+// Launch of the persistent kernel (bn_max 16/32/64/128, head_dim 64/128).
 cudaError_t launch_step_persistent(const StepParams& p, int bn_max, int hd, int grid,
                                    cudaStream_t s, bool cooperative);
 cudaError_t step_persistent_set_attributes();

@@ -57,7 +57,9 @@ def test_ranges_cover_chunks_and_owners_end_ranges(plan, name, sms):
     p = plan(mtiles, K, 16, sms)
     kc, cpc, grid = p["kchunks"], p["cpc"], p["grid"]
     total = mtiles * kc
-    assert kc == -(-K // 64)
+    # even chunk counts: every tile and every range starts on a pair of chunks
+    assert kc == -(-(-(-K // 64)) // 2) * 2
+    assert kc % 2 == 0 and cpc % 2 == 0
     assert grid <= sms
     ranges = [(c * cpc, min(total, (c + 1) * cpc)) for c in range(grid)]
     assert ranges[0][0] == 0 and ranges[-1][1] == total
