@@ -56,8 +56,9 @@ int cllm_test_phase_stamps(cllm_ctx *ctx, unsigned long long *out, int cap, cons
  * (barrier seen), 1 MMA issuer done with the phase (GEMM phases), 2 arrival
  * at the grid barrier, 3-5 the epilogue's last segment (accumulator ready,
  * after the split-K ticket, done), 6 producer enters the phase, 8 producer
- * done, 10/11 first/last stage arrival at the MMA, 12 largest gap between
- * arrivals (ns); slots 7 and 9 are unused (0).  Then 256 * G traced arrivals
+ * done, 7 the split-K owner's partials summed (its last segment), 10/11
+ * first/last stage arrival at the MMA, 12 largest gap between arrivals (ns);
+ * slot 9 is unused (0).  Then 256 * G traced arrivals
  * (see cllm_test_set_trace_phase).  G = SM count.  Returns the number of
  * values, (13 * P + 256) * G. */
 int cllm_test_cta_stamps(cllm_ctx *ctx, unsigned long long *out, long long cap);

@@ -252,7 +252,7 @@ class Engine:
         if record_cap > 0:
             traj = np.zeros((record_cap, B, n), dtype=np.int32)
             _check(self._lib.cllm_decode_read_trajectory(self._h, _ip(traj)),
-                   "cllm_decode_read_trajectory", "cllm_decode_read_stats")
+                   "cllm_decode_read_trajectory")
             return out, its, traj
         return out, its
 

@@ -506,6 +506,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
           }
           epi_sync();
         }
+        if (dbg && ch == 0) e.dbg[4 * e.dbg_stride + cta] = globaltimer_ns();
         epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
       }
       tc_fence_before();

@@ -70,7 +70,7 @@ struct EpiArgs {
   int* err;
   // optional timing of the epilogue's last segment (persistent kernel
   // profiling): dbg[k * dbg_stride + cta], k = 0 accumulator ready, 1 after
-  // the arrival ticket, 2 epilogue done
+  // the arrival ticket, 2 epilogue done, 4 split-K partials summed (owner)
   unsigned long long* dbg;
   long long dbg_stride;
 };
