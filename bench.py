@@ -196,13 +196,23 @@ def gateup_bytes(cfg, T):
 # oracle (CPU) baseline: bounded sample of the same workload
 # ----------------------------------------------------------------------------------------
 
-def oracle_sample(cfg, n, steps=3, warmup=0, layers=2, seed=0):
+def host_cores():
+    """Cores this process may run on (its CPU affinity set)."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except (AttributeError, OSError):
+        return os.cpu_count() or 1
+
+
+def oracle_sample(cfg, n, steps=3, warmup=0, layers=2, seed=0, plen=128, threads=(None,)):
     """Time the oracle's Jacobi iteration (n rows) of a 7B-shaped decoder on the
     host cores.  Sample: the first `layers` decoder layers plus the LM head,
-    over a 16-token prompt, every iteration from the same committed state (a
-    fresh guess block each time); the time is scaled to the full depth by
-    weight bytes (weight streaming dominates the oracle's cost; the prompt
-    length changes it by < 1%)."""
+    over a `plen`-token prompt (the workload's; prefilled on every core), every
+    iteration from the same committed state (a fresh guess block each time),
+    timed with each thread count in `threads` (None: the oracle's default).
+    Returns, per thread count, the measured time per sampled iteration and,
+    separately, the factor that scales it to the full depth by weight bytes
+    (weight streaming dominates the oracle's cost)."""
     from dataclasses import replace
 
     from oracle import oracle as orc
@@ -211,54 +221,179 @@ def oracle_sample(cfg, n, steps=3, warmup=0, layers=2, seed=0):
     sub = replace(cfg, n_layers=Ls)
     w = syn.make_weights(sub, seed=seed, device="cpu")
     om = orc.OracleModel(orc.OracleArch(**syn.oracle_arch_kwargs(sub)), w, orc.ORC_BF16)
-    prompt = syn.make_prompts(cfg.vocab, [16], seed=1)[0]
-    sess = om.session(16 + n + 8)
+    prompt = syn.make_prompts(cfg.vocab, [plen], seed=1)[0]
+    sess = om.session(plen + n + 8)
     head, _, _ = orc.prefill(sess, prompt)
     L = len(prompt)
-    times, acc = [], []
-    for it in range(warmup + steps):
-        blk = [head] + [orc.guess_token(2, 0, it, k, cfg.vocab) for k in range(1, n)]
-        t0 = time.perf_counter()
-        st = orc.jacobi_step(sess, blk, L)
-        dt = time.perf_counter() - t0
-        if it >= warmup:
-            times.append(dt)
-            acc.append(st.accepted)
     lw = 2 * (cfg.d_model * cfg.vocab)
     per_layer_bytes = (step_bytes(sub, 1, n, L) - lw) / Ls
     scale = (cfg.n_layers * per_layer_bytes + lw) / (Ls * per_layer_bytes + lw)
-    total = sum(times) * scale
-    return {
-        "step_s": total / len(times), "accepted_total": sum(acc), "steps": len(times),
-        "cores": orc.num_threads(),
-        "sample": (f"oracle Jacobi iteration, n={n}, layers 1-{Ls} of {cfg.n_layers} + LM head of the "
-                   f"{cfg.name} shape, 16-token prompt, {len(times)} iteration(s) from one committed "
-                   f"state, time scaled x{scale:.2f} to {cfg.n_layers} layers by weight bytes"),
-    }
+    prev = orc.num_threads()
+    out = []
+    try:
+        for th in threads:
+            if th:
+                orc.set_num_threads(th)
+            used = orc.num_threads()
+            times, acc = [], []
+            for it in range(warmup + steps):
+                blk = [head] + [orc.guess_token(2, 0, it, k, cfg.vocab) for k in range(1, n)]
+                t0 = time.perf_counter()
+                st = orc.jacobi_step(sess, blk, L)
+                dt = time.perf_counter() - t0
+                if it >= warmup:
+                    times.append(dt)
+                    acc.append(st.accepted)
+            sample_s = sum(times) / len(times)
+            out.append({
+                "sample_s_per_step": sample_s, "scale_to_full_depth": scale, "step_s": sample_s * scale,
+                "accepted_total": sum(acc), "steps": len(times), "threads": used,
+                "sample": (f"oracle Jacobi iteration, n={n}, layers 1-{Ls} of {cfg.n_layers} + LM head "
+                           f"of the {cfg.name} shape, {plen}-token prompt, {len(times)} iteration(s) from "
+                           f"one committed state on {used} thread(s); measured time per sampled "
+                           f"iteration {sample_s * 1e3:.1f} ms, scaled x{scale:.2f} to {cfg.n_layers} "
+                           f"layers by weight bytes")})
+    finally:
+        orc.set_num_threads(prev)
+        sess.close()
+    return out
+
+
+def oracle_tiny_decodes(max_new=64, n=8):
+    """Wall time of the oracle's full decodes of the tiny fp32 configuration
+    (32-token prompt): greedy AR and Jacobi (refill policy, block n)."""
+    from oracle import oracle as orc
+    from paper_2403_00835_gb300 import synthetic as syn
+    cfg = syn.TINY
+    w = syn.make_weights(cfg, seed=0, device="cpu")
+    om = orc.OracleModel(orc.OracleArch(**syn.oracle_arch_kwargs(cfg)), w, orc.ORC_F32)
+    prompt = syn.make_prompts(cfg.vocab, [32], seed=1)[0]
+    t0 = time.perf_counter()
+    ar = orc.ar_decode(om, prompt, max_new)
+    t1 = time.perf_counter()
+    jr = orc.jacobi_decode(om, prompt, n, max_new, seed=2)
+    t2 = time.perf_counter()
+    return {"config": "tiny fp32 (2 layers, d 256, vocab 2048), prompt 32, max_new 64",
+            "ar_s": t1 - t0, "ar_tokens_per_s": len(ar.tokens) / (t1 - t0),
+            "jacobi_n8_s": t2 - t1, "jacobi_n8_tokens_per_s": len(jr.tokens) / (t2 - t1),
+            "jacobi_n8_iterations": jr.iterations, "threads": orc.num_threads()}
+
+
+def cpu_baseline_entry(cfg, n, plen):
+    """The bench line's cpu_baseline: the oracle on every host core and on one
+    core (7B-shaped sample), plus full tiny-config decodes."""
+    cores = host_cores()
+    cb, one = oracle_sample(cfg, n, steps=2, warmup=0, layers=2, plen=plen, threads=(cores, 1))
+    value = cb["accepted_total"] / (cb["step_s"] * cb["steps"])
+    return {"value": value, "unit": "tokens/s", "cores": cb["threads"], "kind": "oracle",
+            "sample": cb["sample"], "host_cores": cores,
+            "sample_ms_per_step": cb["sample_s_per_step"] * 1e3,
+            "scale_to_full_depth": cb["scale_to_full_depth"],
+            "extrapolated_ms_per_step": cb["step_s"] * 1e3,
+            "one_core": {"value": one["accepted_total"] / (one["step_s"] * one["steps"]),
+                         "sample_ms_per_step": one["sample_s_per_step"] * 1e3,
+                         "extrapolated_ms_per_step": one["step_s"] * 1e3, "cores": 1},
+            "tiny_full_decodes": oracle_tiny_decodes()}
 
 
 # ----------------------------------------------------------------------------------------
 
 def run_reference(args, rank):
+    """The reference arm: the oracle (this tier has no reference implementation
+    to install), timed as it stands on the host cores over a bounded sample of
+    the workload -- every step one Jacobi iteration of the first 2 of the 32
+    layers plus the LM head.  ms_per_step is the measured time of that sampled
+    step; value extrapolates it to the full depth by weight bytes (the factor
+    is reported as scale_to_full_depth)."""
     from paper_2403_00835_gb300 import synthetic as syn
     if rank != 0:
         return 0  # under torchrun only rank 0 runs the CPU reference
     cname, B, lens, n, max_new = WORKLOADS[args.workload]
     cfg = syn.CONFIGS[cname]
-    res = oracle_sample(cfg, n, steps=args.steps, warmup=args.warmup, layers=args.cpu_layers)
-    step_s = res["step_s"]
-    value = res["accepted_total"] / (step_s * res["steps"])
+    cores = host_cores()
+    res = oracle_sample(cfg, n, steps=args.steps, warmup=args.warmup, layers=args.cpu_layers,
+                        plen=lens[0] if lens[0] == lens[1] else 128, threads=(cores,))[0]
+    value = res["accepted_total"] / (res["step_s"] * res["steps"])
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": res["sample_s_per_step"] * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(args.workload),
-        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": res["cores"], "kind": "oracle",
-                         "sample": res["sample"]},
+        "scale_to_full_depth": res["scale_to_full_depth"],
+        "extrapolated_ms_per_step": res["step_s"] * 1e3,
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": res["threads"], "kind": "oracle",
+                         "sample": res["sample"], "host_cores": cores},
         "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
     return 0
+
+
+def decode_loop_ms(eng, nblk, max_new, steps, warmup, seed, stream, dist=None):
+    """`steps` iterations of the device-resident decode loop after `warmup`
+    untimed ones, timed with CUDA events on the engine's stream; a decode that
+    reaches max_new is restarted from the prefill (inside the timed region).
+    Returns (ms, committed tokens, restarts)."""
+    import torch
+
+    def run(iters):
+        committed, restarts = 0, 0
+        left = iters
+        while left > 0:
+            it, c = eng.decode_run(left)
+            left -= it
+            committed += c
+            if left > 0:
+                eng.decode_begin(nblk, max_new, seed=seed)
+                restarts += 1
+        return committed, restarts
+
+    eng.decode_begin(nblk, max_new, seed=seed)
+    run(warmup)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    committed, restarts = run(steps)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1), committed, restarts
+
+
+def extra_workload(name, steps, warmup, local, weights=None):
+    """Step time of another workload of the metric's range (Jacobi and the
+    same-kernel AR step), for the bench line's extra keys.  `weights` reuses
+    device weights of the same configuration."""
+    import numpy as np
+    import torch
+
+    from paper_2403_00835_gb300 import synthetic as syn
+    from paper_2403_00835_gb300.cllm import Engine
+    cname, B, lens_rng, n, max_new = WORKLOADS[name]
+    cfg = syn.CONFIGS[cname]
+    lens = [lens_rng[0]] * B if lens_rng[0] == lens_rng[1] else syn.ragged_lens(B, *lens_rng, seed=1)
+    prompts = syn.make_prompts(cfg.vocab, lens, seed=1)
+    w = weights if weights is not None else syn.make_weights(cfg, seed=0, device=f"cuda:{local}")
+    stream = torch.cuda.current_stream()
+    eng = Engine(cfg, w, max_batch=B, max_seq=max(lens) + max_new + n + 16, max_block=n, stream=stream)
+    try:
+        eng.prefill(prompts)
+        with ClockSampler(local) as clk:
+            ms_j, com_j, _ = decode_loop_ms(eng, n, max_new, steps, warmup, 2, stream)
+            ms_a, _, _ = decode_loop_ms(eng, 1, max_new, steps, warmup, 2, stream)
+        persistent = bool(eng.uses_persistent(n))
+    finally:
+        eng.close()
+    hbm, _, peak_kind = measured_peaks()
+    ms_step, ms_ar = ms_j / steps, ms_a / steps
+    sb = step_bytes(cfg, B, n, float(np.mean(lens)) + max_new / 2)
+    return {"workload": workload_config(name)["workload"], "steps": steps, "warmup": warmup,
+            "ms_per_step": ms_step, "ar_ms_per_step": ms_ar, "jacobi_over_ar_step": ms_step / ms_ar,
+            "tokens_per_s": com_j / (ms_j / 1e3),
+            "step_hbm_roofline": {"bytes": sb, "achieved_gbs": sb / (ms_step / 1e3) / 1e9, "peak_gbs": hbm,
+                                  "frac": sb / (ms_step / 1e3) / 1e9 / hbm, "peak_kind": peak_kind},
+            "path": "persistent kernel" if persistent else "per-GEMM kernels", "clocks": clk.summary()}
 
 
 def workload_config(name):
@@ -296,31 +431,7 @@ def run_ours(args, world, rank, local):
     total_new = B * max_new
 
     def timed_loop(nblk, steps, warmup, seed):
-        """`steps` iterations of the device-resident decode loop; a decode that
-        reaches max_new is restarted from the prefill (inside the timed region)."""
-        def run(iters):
-            committed, restarts = 0, 0
-            left = iters
-            while left > 0:
-                it, c = eng.decode_run(left)
-                left -= it
-                committed += c
-                if left > 0:
-                    eng.decode_begin(nblk, max_new, seed=seed)
-                    restarts += 1
-            return committed, restarts
-
-        eng.decode_begin(nblk, max_new, seed=seed)
-        run(warmup)
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize()
-        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        ev0.record(stream)
-        committed, restarts = run(steps)
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        ms = ev0.elapsed_time(ev1)
+        ms, committed, restarts = decode_loop_ms(eng, nblk, max_new, steps, warmup, seed, stream, dist)
         ms, committed = rank_aggregate(dist, "cuda", ms, committed)
         return ms, committed, restarts
 
@@ -417,12 +528,17 @@ def run_ours(args, world, rank, local):
         "gpu_launches": launches_per_iter * args.steps + rs_j,
         "clocks": clocks,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cb = oracle_sample(cfg, n, steps=2, warmup=0, layers=args.cpu_layers)
-        cv = cb["accepted_total"] / (cb["step_s"] * cb["steps"])
-        line["cpu_baseline"] = {"value": cv, "unit": "tokens/s", "cores": cb["cores"], "kind": "oracle",
-                                "sample": cb["sample"]}
     eng.close()
+    if world == 1 and not args.layers and args.workload == "llama7b-n16" and not args.no_extra:
+        # the rest of the metric's range, in the same run and clock record:
+        # the wide block (prompt 512, n = 64) and the ragged coder batch
+        extra_steps = max(3, min(args.steps, 10))
+        line["n64"] = extra_workload("llama7b-n64", extra_steps, args.warmup, local, weights=w)
+        del w
+        torch.cuda.empty_cache()
+        line["coder_b8"] = extra_workload("coder7b-b8", extra_steps, args.warmup, local)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline_entry(cfg, n, lens[0] if len(set(lens)) == 1 else 128)
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
@@ -503,6 +619,8 @@ def main():
     ap.add_argument("--workload", default="llama7b-n16", choices=sorted(WORKLOADS))
     ap.add_argument("--cpu-layers", type=int, default=2)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the extra keys (n64, coder_b8) of the default workload's line")
     ap.add_argument("--layers", type=int, default=0,
                     help="decoder layers (default: the full model); a small count gives a "
                          "same-shape case for profiler captures")

@@ -263,6 +263,11 @@ int cllm_decode_read_stats(cllm_ctx *ctx, cllm_accept_stats *out, int64_t *acc_h
  * slot count mean all).  Results do not depend on it.  Takes effect for
  * graphs captured after the call. */
 #define CLLM_OPT_PARK_SLOTS 3
+/* CLLM_OPT_L2_PAIRS (default 0): in the persistent kernel, while a CTA's weight
+ * ring and tensor-memory slots are full, its producer prefetches the current
+ * phase's next this-many weight pairs (32 KB each) into L2.  0..64.  Results
+ * do not depend on it.  Takes effect for graphs captured after the call. */
+#define CLLM_OPT_L2_PAIRS 2
 int cllm_set_option(cllm_ctx *ctx, int option, int value);
 
 /* 1 if an iteration of width n on the current batch runs as the persistent

@@ -32,6 +32,7 @@ EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "c
            "cllm_decode_read_trajectory", "cllm_decode_read_stats")
 CLLM_OPT_PERSISTENT = 1
 CLLM_OPT_PARK_SLOTS = 3
+CLLM_OPT_L2_PAIRS = 2
 
 
 class CllmError(RuntimeError):
@@ -304,6 +305,9 @@ class Engine:
 
     def set_persistent(self, on: bool):
         _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PERSISTENT, 1 if on else 0), "cllm_set_option")
+
+    def set_l2_pairs(self, pairs: int):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_L2_PAIRS, int(pairs)), "cllm_set_option")
 
     def set_park_slots(self, tiles: int):
         _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PARK_SLOTS, int(tiles)), "cllm_set_option")

@@ -187,6 +187,7 @@ struct cllm_ctx {
   };
   bool persistent = true;  // one persistent kernel per iteration where supported
   int park_slots = 0;  // persistent kernel: tensor-memory park slots in use (0: all)
+  int l2_pairs = 0;    // persistent kernel: weight pairs prefetched into L2 when the ring is full
   std::vector<unsigned long long> last_stamps;  // last profiled persistent iteration
   std::vector<std::string> last_phase_names;
   std::vector<unsigned long long> last_cta_stamps;
@@ -764,6 +765,7 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   sa.map_attn_v = mapA + 1;
   sa.map_attn_q = mapA + 2;
   sa.park_limit = c->park_slots;
+  sa.l2_ahead = c->l2_pairs;
   sa.err = c->err;
   return CLLM_OK;
 }
@@ -786,7 +788,7 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                                                  : 0,
                              (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0) |
                                  (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0),
-                             c->persistent ? 1 : 0, c->park_slots);
+                             c->persistent ? 1 : 0, c->park_slots * 4096 + c->l2_pairs);
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
     *out = &it->second;
@@ -1647,6 +1649,11 @@ extern "C" int cllm_set_option(cllm_ctx* c, int option, int value) {
   if (!c) return CLLM_EINVAL;
   if (option == CLLM_OPT_PERSISTENT) {
     c->persistent = value != 0;
+    return CLLM_OK;
+  }
+  if (option == CLLM_OPT_L2_PAIRS) {
+    if (value < 0 || value > 64) return CLLM_EINVAL;
+    c->l2_pairs = value;
     return CLLM_OK;
   }
   if (option == CLLM_OPT_PARK_SLOTS) {

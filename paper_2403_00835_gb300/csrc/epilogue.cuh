@@ -420,11 +420,13 @@ __device__ inline void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
     float v1 = -INFINITY, v2 = -INFINITY;
     int i1 = INT_MAX;
     if (t < e.T) {
-      for (int mt0 = part; mt0 < e.am_mtiles; mt0 += 64) {
-        float w1[8], w2[8];
-        int j1[8];
+      // every tile of a 256-tile vocabulary in one round trip (32 loads of
+      // each kind in flight per thread)
+      for (int mt0 = part; mt0 < e.am_mtiles; mt0 += 256) {
+        float w1[32], w2[32];
+        int j1[32];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {  // eight tiles' loads in flight at once
+        for (int u = 0; u < 32; ++u) {
           const int mt = mt0 + 8 * u;
           if (mt < e.am_mtiles) {
             const float* p = e.am_part + (static_cast<size_t>(mt) * e.ldt + t) * 3;
@@ -438,7 +440,7 @@ __device__ inline void epi_argmax_finish(const EpiArgs& e, int r, EpiSmem& s) {
           }
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) am_merge(v1, i1, v2, w1[u], j1[u], w2[u]);
+        for (int u = 0; u < 32; ++u) am_merge(v1, i1, v2, w1[u], j1[u], w2[u]);
       }
     }
 #pragma unroll

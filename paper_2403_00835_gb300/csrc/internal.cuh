@@ -226,6 +226,9 @@ struct StepArgs {
   // tensor-memory park slots the weight stream may fill ahead of the MMAs
   // (0: all the kernel has)
   int park_limit;
+  // weight pairs of the current phase prefetched into L2 while the weight
+  // ring is full (0: none)
+  int l2_ahead;
   int* err;
 };
 

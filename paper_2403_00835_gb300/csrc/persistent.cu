@@ -208,13 +208,44 @@ __device__ __forceinline__ void pk_load_a_chunk(uint8_t* dst, uint64_t* bar, con
   }
 }
 
+template <int KIND>
+__device__ __forceinline__ void pk_prefetch_chunk(const GemmArgs& g, const CUtensorMap* mA0,
+                                                  const CUtensorMap* mA1, const CUtensorMap* mA2,
+                                                  int c) {
+  const int u = c / g.kchunks, k = c - u * g.kchunks;
+  const int mt = u / g.ntiles;
+  if (KIND == EPI_GATEUP) {
+    tma_prefetch_l2_2d(mA0, k * kBK, mt * 64);
+    tma_prefetch_l2_2d(mA1, k * kBK, mt * 64);
+  } else if (KIND == EPI_QKV) {
+    const int row = mt * kBM;
+    if (row < g.rows_q)
+      tma_prefetch_l2_2d(mA0, k * kBK, row);
+    else if (row < g.rows_qk)
+      tma_prefetch_l2_2d(mA1, k * kBK, row - g.rows_q);
+    else
+      tma_prefetch_l2_2d(mA2, k * kBK, row - g.rows_qk);
+  } else {
+    tma_prefetch_l2_2d(mA0, k * kBK, mt * kBM);
+  }
+}
+
 template <int KIND, class PC>
 __device__ bool pk_produce_a(const PkPipe& P, int& ia, const GemmArgs& g, const CUtensorMap* mA0,
-                             const CUtensorMap* mA1, const CUtensorMap* mA2, int c0, int c1) {
+                             const CUtensorMap* mA1, const CUtensorMap* mA2, int c0, int c1,
+                             int l2_ahead) {
   constexpr int S = PC::SA;
   const uint64_t pol_w = l2_policy_evict_first();
+  int pf = c0;  // next chunk of this phase to prefetch into L2
   for (int c = c0; c < c1; c += kPairChunks, ++ia) {
     const int st = ia % S;
+    if (l2_ahead > 0 && !mbar_test_wait(&P.aempty[st], ((ia / S) & 1) ^ 1)) {
+      // the ring is full (shared and tensor memory hold every tile they
+      // can): fetch the phase's next tiles into L2 meanwhile
+      if (pf < c + kPairChunks) pf = c + kPairChunks;
+      for (; pf < c1 && pf < c + kPairChunks * (1 + l2_ahead); ++pf)
+        pk_prefetch_chunk<KIND>(g, mA0, mA1, mA2, pf);
+    }
     if (!mbar_wait(&P.aempty[st], ((ia / S) & 1) ^ 1, P.abort)) return false;
     if (S > kMaxWeightPairs && ia >= kMaxWeightPairs) {  // at most kMaxWeightPairs in flight
       const int o = ia - kMaxWeightPairs;  // (its stage is not reused before this pair)
@@ -399,7 +430,7 @@ __device__ bool pk_mma(const PkPipe& P, PkMmaState& q, int& acc, uint32_t& accph
 // (TMA issue, mbarrier operations) would force them to be reloaded.
 template <class PC>
 __device__ bool produce_a_phase(const PkPipe& P, int& ia, const PhaseDesc& ph,
-                                const CUtensorMap* maps, int cta) {
+                                const CUtensorMap* maps, int cta, int l2_ahead) {
   const GemmArgs g = ph.g;
   const CUtensorMap* m0 = maps + ph.map_a0;
   const CUtensorMap* m1 = maps + ph.map_a1;
@@ -407,9 +438,9 @@ __device__ bool produce_a_phase(const PkPipe& P, int& ia, const PhaseDesc& ph,
   int c0, c1;
   cta_range(g, cta, c0, c1);
   switch (ph.epi) {
-    case EPI_QKV: return pk_produce_a<EPI_QKV, PC>(P, ia, g, m0, m1, m2, c0, c1);
-    case EPI_GATEUP: return pk_produce_a<EPI_GATEUP, PC>(P, ia, g, m0, m1, m2, c0, c1);
-    default: return pk_produce_a<EPI_RESID, PC>(P, ia, g, m0, m1, m2, c0, c1);
+    case EPI_QKV: return pk_produce_a<EPI_QKV, PC>(P, ia, g, m0, m1, m2, c0, c1, l2_ahead);
+    case EPI_GATEUP: return pk_produce_a<EPI_GATEUP, PC>(P, ia, g, m0, m1, m2, c0, c1, l2_ahead);
+    default: return pk_produce_a<EPI_RESID, PC>(P, ia, g, m0, m1, m2, c0, c1, l2_ahead);
   }
 }
 
@@ -474,7 +505,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
         unsigned long long* cs =
             A.cta_stamps != nullptr ? A.cta_stamps + static_cast<size_t>(p) * G + cta : nullptr;
         if (cs != nullptr) cs[6 * PG] = globaltimer_ns();
-        const bool ok = produce_a_phase<PC>(K, ia, ph, PRM.maps, cta);
+        const bool ok = produce_a_phase<PC>(K, ia, ph, PRM.maps, cta, A.l2_ahead);
         if (cs != nullptr) cs[8 * PG] = globaltimer_ns();
         if (!ok) break;
       }
