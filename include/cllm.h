@@ -257,7 +257,7 @@ int cllm_decode_read_stats(cllm_ctx *ctx, cllm_accept_stats *out, int64_t *acc_h
  */
 #define CLLM_OPT_PERSISTENT 1
 /* CLLM_OPT_PARK_SLOTS (default 0 = all): in the persistent kernel, the weight
- * tiles (16 KB each) a CTA may hold in tensor memory ahead of its MMAs.  The
+ * pairs (32 KB each) a CTA may hold in tensor memory ahead of its MMAs.  The
  * weight stream runs ahead of the grid barriers into these slots, so HBM keeps
  * streaming while a phase drains; 1..64 limits it (values above the kernel's
  * slot count mean all).  Results do not depend on it.  Takes effect for
@@ -268,6 +268,13 @@ int cllm_decode_read_stats(cllm_ctx *ctx, cllm_accept_stats *out, int64_t *acc_h
  * phase's next this-many weight pairs (32 KB each) into L2.  0..64.  Results
  * do not depend on it.  Takes effect for graphs captured after the call. */
 #define CLLM_OPT_L2_PAIRS 2
+/* CLLM_OPT_DATAFLOW (default 1): in the persistent kernel, attention and the
+ * O projection start on per-tile completion flags instead of grid barriers:
+ * an attention item waits for its head's Q, K and V tiles of the QKV GEMM, a
+ * pair of O-projection K chunks for its heads' attention outputs.  0 = grid
+ * barriers before both.  Results do not depend on it.  Takes effect for
+ * graphs captured after the call. */
+#define CLLM_OPT_DATAFLOW 4
 int cllm_set_option(cllm_ctx *ctx, int option, int value);
 
 /* 1 if an iteration of width n on the current batch runs as the persistent

@@ -33,6 +33,7 @@ EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "c
 CLLM_OPT_PERSISTENT = 1
 CLLM_OPT_PARK_SLOTS = 3
 CLLM_OPT_L2_PAIRS = 2
+CLLM_OPT_DATAFLOW = 4
 
 
 class CllmError(RuntimeError):
@@ -311,6 +312,9 @@ class Engine:
 
     def set_park_slots(self, tiles: int):
         _check(self._lib.cllm_set_option(self._h, CLLM_OPT_PARK_SLOTS, int(tiles)), "cllm_set_option")
+
+    def set_dataflow(self, on: bool):
+        _check(self._lib.cllm_set_option(self._h, CLLM_OPT_DATAFLOW, 1 if on else 0), "cllm_set_option")
 
     def uses_persistent(self, n: int) -> bool:
         r = self._lib.cllm_uses_persistent(self._h, n)

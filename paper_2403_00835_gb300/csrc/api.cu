@@ -184,10 +184,12 @@ struct cllm_ctx {
     std::vector<void*> bufs;           // device tables owned by the graph
     unsigned long long* stamps = nullptr;
     unsigned long long* cta_stamps = nullptr;
+    size_t bar_bytes = 64;             // grid-barrier counter and completion flags
   };
   bool persistent = true;  // one persistent kernel per iteration where supported
   int park_slots = 0;  // persistent kernel: tensor-memory park slots in use (0: all)
   int l2_pairs = 0;    // persistent kernel: weight pairs prefetched into L2 when the ring is full
+  bool dataflow = true;  // persistent kernel: attention and O open on completion flags
   std::vector<unsigned long long> last_stamps;  // last profiled persistent iteration
   std::vector<std::string> last_phase_names;
   std::vector<unsigned long long> last_cta_stamps;
@@ -630,6 +632,17 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   f.n = n;
   f.qtiles = qtiles;
   f.n_qtiles = n_qtiles;
+  // grid-barrier counter (16 words) then, per layer, the QKV tile flags and
+  // the per-head attention counts; zeroed with the counter every launch
+  const int Mqkv = c->dq + 2 * c->dkv;
+  const int n_flags_layer = Mqkv / kBM + c->H;
+  const size_t bar_bytes = 64 + sizeof(unsigned) * static_cast<size_t>(NL) * n_flags_layer;
+  void* bar_d = nullptr;
+  if (lib_malloc(&bar_d, bar_bytes) != cudaSuccess) return CLLM_ENOMEM;
+  ge.bufs.push_back(bar_d);
+  if (cudaMemset(bar_d, 0, bar_bytes) != cudaSuccess) return CLLM_ECUDA;
+  ge.bar_bytes = bar_bytes;
+  unsigned* flags = static_cast<unsigned*>(bar_d) + 16;
   std::vector<PhaseDesc> ph;
   auto gemm_phase = [&](int epi, int m0, int m1, int m2, int mb, int mtiles, int M, int K,
                         EpiArgs e) {
@@ -652,7 +665,6 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     d.kind = PH_EMBED;
     ph.push_back(d);
   }
-  const int Mqkv = c->dq + 2 * c->dkv;
   for (int l = 0; l < NL; ++l) {
     const LayerW& L = c->layers[l];
     const size_t kvoff = static_cast<size_t>(l) * c->layer_kv_elems * c->esz;
@@ -663,12 +675,22 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     e.q_out = c->q;
     e.k_cache = kl;
     e.v_cache = vl;
+    unsigned* qkv_done = flags + static_cast<size_t>(l) * n_flags_layer;
+    unsigned* head_done = qkv_done + Mqkv / kBM;
+    if (c->dataflow) e.tile_done = qkv_done;
     gemm_phase(EPI_QKV, 7 * l, 7 * l + 1, 7 * l + 2, mapB, Mqkv / kBM, Mqkv, c->d, e);
+    const int qkv_ntiles = ph.back().g.ntiles;
     PhaseDesc at{};
     at.kind = PH_ATTN;
     at.k_cache = kl;
     at.v_cache = vl;
     at.kv_row0 = static_cast<int>(static_cast<size_t>(l) * c->layer_kv_elems / c->hd);
+    if (c->dataflow) {
+      at.no_barrier = 1;
+      at.qkv_done = qkv_done;
+      at.head_done = head_done;
+      at.flag_target = qkv_ntiles;
+    }
     ph.push_back(at);
     e = base_epi(c, T);
     e.x = c->x;
@@ -676,6 +698,11 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
     e.gnext = L.mlp_norm;
     e.ssq_out = c->ssq;
     gemm_phase(EPI_RESID, 7 * l + 3, 7 * l + 3, 7 * l + 3, mapB + 1, c->d / kBM, c->d, c->dq, e);
+    if (c->dataflow) {
+      ph.back().no_barrier = 1;
+      ph.back().head_done = head_done;
+      ph.back().flag_target = n_qtiles;
+    }
     e = base_epi(c, T);
     e.ssq_in = c->ssq;
     e.h_out = c->h;
@@ -729,11 +756,10 @@ int build_persistent(cllm_ctx* c, int mode, int B, int n, const int2* qtiles, in
   for (size_t i = 0; i < maps.size(); ++i) prm.maps[i] = maps[i];
   void* ph_d = upload(ph.data(), ph.size() * sizeof(PhaseDesc));
   void* tk_d = upload(nullptr, static_cast<size_t>(n_qtiles) * c->H * sizeof(int) + 16);
-  void* bar_d = upload(nullptr, 64);
   void* st_d = upload(nullptr, (5 * ph.size() + 1) * sizeof(unsigned long long));
   void* cst_d = upload(nullptr, (kCtaStampSlots * ph.size() + kTraceCap) * c->sms *
                                     sizeof(unsigned long long));
-  if (!ph_d || !tk_d || !bar_d || !st_d || !cst_d) return CLLM_ENOMEM;
+  if (!ph_d || !tk_d || !st_d || !cst_d) return CLLM_ENOMEM;
   ge.cta_stamps = static_cast<unsigned long long*>(cst_d);
   if (c->profiling) {
     // epilogue stamps k = 3..5 of the per-CTA stamp array
@@ -788,7 +814,8 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                                                  : 0,
                              (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0) |
                                  (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0),
-                             c->persistent ? 1 : 0, c->park_slots * 4096 + c->l2_pairs);
+                             c->persistent ? 1 : 0,
+                             (c->park_slots * 4096 + c->l2_pairs) * 2 + (c->dataflow ? 1 : 0));
   auto it = c->graphs.find(key);
   if (it != c->graphs.end()) {
     *out = &it->second;
@@ -826,7 +853,7 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
     cudaGraph_t g = nullptr;
     cudaError_t e = cudaStreamBeginCapture(c->stream, cudaStreamCaptureModeThreadLocal);
     if (e != cudaSuccess) return cuda_fail(e, "begin capture (persistent)");
-    e = cudaMemsetAsync(sa.bar, 0, 64, c->stream);
+    e = cudaMemsetAsync(sa.bar, 0, ge.bar_bytes, c->stream);
     if (e == cudaSuccess && prof) {
       // first-of slots start at all-ones (atomicMin), last-of slots at zero
       const size_t P = ge.n_phases;
@@ -1659,6 +1686,10 @@ extern "C" int cllm_set_option(cllm_ctx* c, int option, int value) {
   if (option == CLLM_OPT_PARK_SLOTS) {
     if (value < -1 || value > 64) return CLLM_EINVAL;
     c->park_slots = value;
+    return CLLM_OK;
+  }
+  if (option == CLLM_OPT_DATAFLOW) {
+    c->dataflow = value != 0;
     return CLLM_OK;
   }
   return CLLM_EINVAL;

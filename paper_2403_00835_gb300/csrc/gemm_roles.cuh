@@ -404,6 +404,15 @@ __device__ __forceinline__ void tmem_ld_sum_cfg(uint32_t taddr, int ch, int bn, 
   for (int j = 0; j < kEpiCols; ++j) v[j] += vlo[j];
 }
 
+// Persistent kernel: publish a finished output tile (its stores are read next
+// by other CTAs, some through TMA) on its completion flag.
+__device__ __forceinline__ void epi_publish(const EpiArgs& e, int mt, int r) {
+  if (e.tile_done == nullptr) return;
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  epi_sync();
+  if (r == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(e.tile_done + mt) : "memory");
+}
+
 template <int KIND, class Cfg>
 __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const GemmArgs& g,
                             const EpiArgs& e, int c0, int c1, int cta, EpiSmem& es) {
@@ -454,6 +463,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
           for (int j = 0; j < kEpiCols; ++j) mypart[(ch * kEpiCols + j) * kBM + r] = v[j];
         }
       }
+      if (nc == 1) epi_publish(e, mt, r);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&P.tempty[acc]);
@@ -509,10 +519,13 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
         if (dbg && ch == 0) e.dbg[4 * e.dbg_stride + cta] = globaltimer_ns();
         epi_apply<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, v, r, es, &pre);
       }
+      // (the count is reset before the tile is published: a later phase that
+      // the flag opens may count on the same ticket)
+      if (r == 0) g.tickets[u] = 0;
+      epi_publish(e, mt, r);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&P.tempty[acc]);
-      if (r == 0) g.tickets[u] = 0;
       if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
     }
     if (dbg) e.dbg[2 * e.dbg_stride + cta] = globaltimer_ns();

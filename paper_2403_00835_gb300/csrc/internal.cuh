@@ -68,6 +68,9 @@ struct EpiArgs {
   float* logits;  // optional debug [T][V]
   int V;
   int* err;
+  // persistent kernel: completion flag of each finished output tile (QKV:
+  // released after the tile's Q/K/V stores; null: none)
+  unsigned* tile_done;
   // optional timing of the epilogue's last segment (persistent kernel
   // profiling): dbg[k * dbg_stride + cta], k = 0 accumulator ready, 1 after
   // the arrival ticket, 2 epilogue done, 4 split-K partials summed (owner)
@@ -201,6 +204,17 @@ struct PhaseDesc {
   const void* k_cache;
   const void* v_cache;
   int kv_row0;  // attention: the layer's first row in the K/V cache tensor maps
+  // Dependencies narrower than the grid barrier (no_barrier = 1: the phase
+  // does not wait for it).  Attention: the item of head h waits until the
+  // QKV tile flags qkv_done[] of h's Q, K and V tiles reach flag_target (the
+  // QKV GEMM's column tiles), and adds 1 to head_done[h] for every query tile
+  // whose output it completes.  O projection: a pair of K chunks waits for
+  // its heads' head_done[] to reach flag_target (the query tiles) and for
+  // this CTA's attention phase to end.
+  int no_barrier;
+  const unsigned* qkv_done;
+  unsigned* head_done;
+  int flag_target;
 };
 
 struct StepArgs {
@@ -238,9 +252,9 @@ constexpr int kMaxQTilesStep = 256;  // query tiles of one iteration (persistent
 
 // Tensor maps travel by value in the kernel's parameter space (TMA reads
 // descriptors there as it does for per-GEMM kernels): 7 per layer + the LM
-// head + 3 activation maps + the attention's K, V and Q maps, at most 32
-// layers (29.6 KB of the 32 KB limit).
-constexpr int kMaxStepMaps = 7 * 32 + 7;
+// head + 4 activation maps + the attention's K, V and Q maps, at most 32
+// layers (29.7 KB of the 32 KB limit).
+constexpr int kMaxStepMaps = 7 * 32 + 8;
 struct StepParams {
   StepArgs a;
   CUtensorMap maps[kMaxStepMaps];

@@ -89,7 +89,7 @@ struct PersistCfg {
   static constexpr int BN = BNMAX;
   static constexpr int PARK_COL0 = NACC * ACC_COLS;
   static constexpr int NPARK = (kTmemCols - PARK_COL0) / kParkCols;
-  static constexpr size_t BAR_FIXED = 8 * (static_cast<size_t>(2 * SB + NPARK + 2 * NACC + 1)) + 16;
+  static constexpr size_t BAR_FIXED = 8 * (static_cast<size_t>(2 * SB + NPARK + 2 * NACC + 2)) + 16;
   static constexpr size_t BUDGET = 227 * 1024 - 256;  // minus the kernel's static shared memory
   static constexpr size_t FIXED0 = 1024 + SHARED_B + EPI_AREA + META_BYTES + BAR_FIXED + 64;
   static constexpr int FIT = static_cast<int>((BUDGET - FIXED0 - 16 * 6) / (A_BYTES + 16));
@@ -114,6 +114,7 @@ struct PkPipe {
   uint64_t* tfull;   // [NACC]
   uint64_t* tempty;  // [NACC]
   uint64_t* drain;
+  uint64_t* attn_free;  // one phase per attention phase: its shared memory is free again
   volatile int* abort;
   uint32_t tmem;
   int park_limit;  // park slots in use (0: none)
@@ -133,7 +134,8 @@ __device__ PkPipe pk_pipe_init(uint8_t* ring, uint8_t* bars) {
   P.tfull = P.pempty + PC::NPARK;
   P.tempty = P.tfull + PC::NACC;
   P.drain = P.tempty + PC::NACC;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(P.drain + 1);
+  P.attn_free = P.drain + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(P.attn_free + 1);
   P.abort = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
@@ -151,6 +153,7 @@ __device__ PkPipe pk_pipe_init(uint8_t* ring, uint8_t* bars) {
       mbar_init(&P.tempty[i], 4);
     }
     mbar_init(P.drain, 1);
+    mbar_init(P.attn_free, 1);
     *P.abort = 0;
     fence_mbar_init();
   }
@@ -259,15 +262,79 @@ __device__ bool pk_produce_a(const PkPipe& P, int& ia, const GemmArgs& g, const 
   return true;
 }
 
+__device__ __forceinline__ unsigned ld_relaxed_gpu(const unsigned* p) {
+  unsigned v;
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+// Smallest of the flags f[i0..i1], up to 8 loads in flight at a time.
+__device__ inline unsigned flags_min(const unsigned* f, int i0, int i1) {
+  unsigned mn = ~0u;
+  for (int b = i0; b <= i1; b += 8) {
+    unsigned v[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) v[j] = (b + j <= i1) ? ld_relaxed_gpu(f + b + j) : ~0u;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) mn = min(mn, v[j]);
+  }
+  return mn;
+}
+
+// Bounded wait until the flags in `idx` (cnt of them, or the range
+// idx[0]..idx[1] when range) reach target; then an acquire fence, and the
+// TMA reads that follow are ordered after the generic stores the flags
+// publish.  Sets *abort when the wait runs out.
+__device__ inline bool wait_flags(const unsigned* f, const int* idx, int cnt, bool range,
+                                  unsigned target, volatile int* abort) {
+  auto low = [&]() -> unsigned {
+    if (range) return flags_min(f, idx[0], idx[1]);
+    unsigned v[3];
+#pragma unroll
+    for (int j = 0; j < 3; ++j) v[j] = j < cnt ? ld_relaxed_gpu(f + idx[j]) : ~0u;
+    return min(v[0], min(v[1], v[2]));
+  };
+  if (low() < target) {
+    const uint64_t t0 = globaltimer_ns();
+    while (low() < target) {
+      if (*abort) return false;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        *abort = 1;
+        return false;
+      }
+      __nanosleep(32);
+    }
+  }
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+  return true;
+}
+
 // ---- producer B: activation pairs, after the phase's grid barrier --------------------
 
+// gate != nullptr (O projection after attention): instead of the grid barrier,
+// the CTA waits for the heads its K chunks cover (columns 64k.. of head
+// 64k/hd) to reach target completions, once its own attention phase has
+// released the shared memory (attn_free, phase attn_phase).
 template <class PC>
 __device__ bool pk_produce_b(const PkPipe& P, int& ib, const GemmArgs& g, const CUtensorMap* mB,
-                             int c0, int c1, const GridDep& dep) {
+                             int c0, int c1, const GridDep& dep, const unsigned* gate,
+                             unsigned target, int hd, int nheads, int attn_phase) {
   constexpr int S = PC::SB;
   if (c0 >= c1) return true;
-  if (!dep.wait(P.abort)) return false;
-  dep.after();
+  if (gate == nullptr) {
+    if (!dep.wait(P.abort)) return false;
+    dep.after();
+  } else {
+    if (!mbar_wait(P.attn_free, attn_phase & 1, P.abort)) return false;
+    const int u0 = c0 / g.kchunks, u1 = (c1 - 1) / g.kchunks;
+    int hr[2] = {0, nheads - 1};
+    if (u0 == u1) {  // (K is padded to whole pairs: clamp to the last head)
+      hr[0] = min(((c0 - u0 * g.kchunks) * kBK) / hd, nheads - 1);
+      hr[1] = min(((c1 - u1 * g.kchunks) * kBK - 1) / hd, nheads - 1);
+    }
+    if (!wait_flags(gate, hr, 2, true, target, P.abort)) return false;
+  }
   const uint64_t pol_x = l2_policy_evict_last();
   const uint32_t b_bytes = 2u * static_cast<uint32_t>(g.bn) * kBK * 2;
   const bool tile_mode = g.ntiles > 1;
@@ -514,15 +581,20 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
   } else if (warp == 6) {
     if (lane == 0) {
       // ---------------- TMA producer: activation tiles ----------------
-      int ib = 0;
+      int ib = 0, attn_phases = 0;
       for (int p = 0; p < A.n_phases; ++p) {
         const PhaseDesc& ph = A.phases[p];
+        if (ph.kind == PH_ATTN) ++attn_phases;
         if (ph.kind != PH_GEMM) continue;
         const GemmArgs g = ph.g;
         int c0, c1;
         cta_range(g, cta, c0, c1);
         const GridDep dep{A.bar, barrier_target(A, p, G)};
-        if (!pk_produce_b<PC>(K, ib, g, PRM.maps + ph.map_b, c0, c1, dep)) break;
+        const unsigned* gate = ph.no_barrier ? ph.head_done : nullptr;
+        const unsigned target = static_cast<unsigned>(ph.flag_target) + (p == A.hold_phase ? 1u : 0u);
+        if (!pk_produce_b<PC>(K, ib, g, PRM.maps + ph.map_b, c0, c1, dep, gate, target, A.attn.hd,
+                              A.attn.H, attn_phases - 1))
+          break;
       }
       pk_ring_drain(K.bfull, PC::SB, ib);
     }
@@ -573,7 +645,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
       const PhaseDesc& ph = A.phases[p];
       const int kind = ph.kind;
       if (kind == PH_ACCEPT && cta != 0) break;
-      if (p > 0) {
+      if (p > 0 && !ph.no_barrier) {
         const GridDep dep{A.bar, barrier_target(A, p, G)};
         if (r == 0) s_flag = dep.wait(P.abort) ? 1 : 0;
         sync();
@@ -612,10 +684,41 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
         const int total = attn_total;
         const AttnTma tma{PRM.maps + A.map_attn_k, PRM.maps + A.map_attn_v, PRM.maps + A.map_attn_q,
                           ph.kv_row0};
+        // an item's head's output is complete once per query tile: publish it
+        // (read next through TMA by the O projection)
+        auto publish_head = [&](int hh) {
+          asm volatile("fence.proxy.async.global;" ::: "memory");
+          sync();
+          if (r == 0)
+            asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ph.head_done + hh) : "memory");
+        };
         for (int item = cta; item < total; item += G) {
+          if (ph.qkv_done != nullptr) {
+            // wait for this item's head's Q, K and V tiles instead of the grid barrier
+            const int qi0 = attn_find_qtile(pre, a.n_qtiles, item);
+            const int hh = (item - pre[qi0]) % a.H;
+            const int kvh = hh / (a.H / a.Hkv);
+            const int dq = a.H * HD, dkv = a.Hkv * HD;
+            const int tq = (hh * HD) / kBM, tk = (dq + kvh * HD) / kBM, tv = (dq + dkv + kvh * HD) / kBM;
+            if (r == 0) {
+              const unsigned tgt = static_cast<unsigned>(ph.flag_target) + (p == A.hold_phase ? 1u : 0u);
+              const int tiles[3] = {tq, tk, tv};
+              s_flag = wait_flags(ph.qkv_done, tiles, 3, false, tgt, P.abort) ? 1 : 0;
+            }
+            sync();
+            const bool ready = s_flag != 0;
+            sync();
+            if (!ready) {
+              ok = false;
+              break;
+            }
+            asm volatile("fence.proxy.async.global;" ::: "memory");  // the item's TMA reads
+          }
           int qi, h;
-          if (attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md, true, &tma))
+          if (attn_mma_item<HD>(a, item, pre, at, r, sync, qi, h, md, true, &tma)) {
+            if (ph.head_done != nullptr) publish_head(h);
             continue;  // output written
+          }
           // the last range of (tile, head) to finish merges the tile's ranges
           sync();
           if (r == 0) {
@@ -628,6 +731,7 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
           if (last) {
             attn_combine_tile<__nv_bfloat16, HD>(a, qi, h, r, md);
             if (r == 0) A.attn_tickets[qi * a.H + h] = 0;
+            if (ph.head_done != nullptr) publish_head(h);
           }
         }
       } else {  // PH_ACCEPT (CTA 0)
@@ -653,6 +757,8 @@ __global__ void __launch_bounds__(kPersistThreads, 1)
               A.cta_stamps[(2 * static_cast<size_t>(A.n_phases) + p) * G + cta] = now;
           }
           asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(A.bar) : "memory");
+          // the attention tile's shared memory is the activation ring again
+          if (kind == PH_ATTN) mbar_arrive(K.attn_free);
         }
       }
     }

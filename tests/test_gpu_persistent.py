@@ -104,3 +104,25 @@ def test_persistent_7b_decode_bit_identical():
             np.testing.assert_array_equal(ia, ib)
     finally:
         eng.close()
+
+
+@pytest.mark.parametrize("n", [1, 16])
+def test_persistent_dataflow_flags_bit_identical(tiny_bf16, n):
+    """Attention and the O projection opened by completion flags (the
+    default) or by grid barriers compute the same logits bit for bit."""
+    cfg, eng = tiny_bf16
+    prompts = syn.make_prompts(cfg.vocab, [32, 17, 45], seed=11)
+    g = syn.make_guesses(cfg.vocab, 3, n, seed=12)
+    out = []
+    try:
+        for flags in (True, False):
+            eng.set_dataflow(flags)
+            eng.prefill(prompts)
+            assert eng.uses_persistent(n)
+            out.append(eng.jacobi_step(g, want_gap=True, want_logits=True))
+    finally:
+        eng.set_dataflow(True)
+    a, b = out
+    np.testing.assert_array_equal(a["logits"], b["logits"])
+    np.testing.assert_array_equal(a["next"], b["next"])
+    np.testing.assert_array_equal(a["accepted"], b["accepted"])
