@@ -354,9 +354,11 @@ def decode_loop_ms(eng, nblk, max_new, steps, warmup, seed, stream, dist=None):
         dist.barrier()
     torch.cuda.synchronize()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push(f"decode_n{nblk}")  # (profiler filter: the timed iterations)
     ev0.record(stream)
     committed, restarts = run(steps)
     ev1.record(stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     return ev0.elapsed_time(ev1), committed, restarts
 
@@ -563,6 +565,9 @@ def run_sweep(args):
         from dataclasses import replace
         cfg = replace(cfg, n_layers=args.layers)
     Ls, ns, Bs = (256, 1024, 4096), (1, 16, 32, 64, 128), (1, 4, 16)
+    if args.point:  # one point of the sweep: L,B,n
+        L0, B0, n0 = (int(v) for v in args.point.split(","))
+        Ls, ns, Bs = (L0,), (n0,), (B0,)
     w = syn.make_weights(cfg, seed=0, device="cuda")
     stream = torch.cuda.current_stream()
     max_new = 256
@@ -584,6 +589,7 @@ def run_sweep(args):
                         eng.decode_begin(n, max_new, seed=2)
                 torch.cuda.synchronize()
                 ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.nvtx.range_push(f"sweep_L{L}_B{B}_n{n}")
                 ev0.record(stream)
                 left, committed = args.steps, 0
                 while left > 0:
@@ -593,6 +599,7 @@ def run_sweep(args):
                     if left > 0:
                         eng.decode_begin(n, max_new, seed=2)
                 ev1.record(stream)
+                torch.cuda.nvtx.range_pop()
                 torch.cuda.synchronize()
                 ms = ev0.elapsed_time(ev1) / args.steps
                 sb = step_bytes(cfg, B, n, L + max_new / 2)
@@ -624,6 +631,8 @@ def main():
     ap.add_argument("--layers", type=int, default=0,
                     help="decoder layers (default: the full model); a small count gives a "
                          "same-shape case for profiler captures")
+    ap.add_argument("--point", default="",
+                    help="with --sweep: only this point, 'L,B,n'")
     ap.add_argument("--sweep", action="store_true",
                     help="step microbenchmark over cache length, block width and batch "
                          "(prints a table instead of the bench line)")
