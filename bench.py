@@ -146,11 +146,12 @@ def emulated_acceptance(workload, B, ms_step):
 
 
 def kernel_sources_digest():
-    """First 16 hex digits of the SHA-256 of the CUDA sources (names and contents)."""
+    """First 16 hex digits of the SHA-256 of the persistent kernel's sources:
+    its translation unit and every CUDA header (names and contents)."""
     h = hashlib.sha256()
     src = os.path.join(ROOT, "paper_2403_00835_gb300", "csrc")
     for name in sorted(os.listdir(src)):
-        if name.endswith((".cu", ".cuh")):
+        if name == "persistent.cu" or name.endswith(".cuh"):
             h.update(name.encode())
             with open(os.path.join(src, name), "rb") as f:
                 h.update(f.read())

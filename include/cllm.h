@@ -312,7 +312,9 @@ int cllm_committed_lengths(cllm_ctx *ctx, int32_t *lens_out);
  * plane), x_rows >= T rounded up to 16 (and >= 256 when T > 256); Y: device
  * fp32 [T][M], accumulated into.  M a multiple of 128, K a multiple of 8.
  * cuda_stream: the cudaStream_t to run on (NULL = the legacy default stream);
- * the call synchronises it before returning.
+ * the call synchronises it before returning, so it can never be captured into
+ * a CUDA graph: on a stream that is capturing it returns CLLM_EUNSUPPORTED
+ * before any work is queued.
  * No memory is allocated: all scratch (split-K partial tiles, arrival tickets,
  * the device error word, epilogue side outputs) lives in one static device
  * array of 8 MiB that each device loading the library holds until exit.  Sizes

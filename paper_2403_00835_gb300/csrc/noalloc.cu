@@ -50,6 +50,12 @@ extern "C" int cllm_gemm_bf16_noalloc(const void* W, const void* X, float* Y, in
   if ((reinterpret_cast<uintptr_t>(W) | reinterpret_cast<uintptr_t>(X) |
        reinterpret_cast<uintptr_t>(Y)) & 15u)
     return CLLM_EINVAL;
+  // the call synchronises its stream and reads the error word back, which a
+  // stream capture cannot hold: refuse before touching the stream
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(static_cast<cudaStream_t>(cuda_stream), &cap) != cudaSuccess)
+    return CLLM_ECUDA;
+  if (cap != cudaStreamCaptureStatusNone) return CLLM_EUNSUPPORTED;
   int dev = 0;
   cudaDeviceProp prop;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess)

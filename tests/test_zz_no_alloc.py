@@ -76,3 +76,26 @@ def test_noalloc_rejects_sizes_beyond_its_scratch():
     rc = lib.cllm_gemm_bf16_noalloc(W.data_ptr(), X2.data_ptr(), out.data_ptr(), M, K, T, T,
                                     ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
     assert rc == -4  # CLLM_ECAPACITY, before any launch
+
+
+def test_noalloc_refuses_stream_capture():
+    """The call synchronises its stream, so it cannot be captured: on a
+    capturing stream it returns CLLM_EUNSUPPORTED and queues nothing."""
+    lib = _lib()
+    W, X2, rows = _inputs(256, 256, 16, seed=3)
+    Y = torch.zeros(16, 256, device="cuda")
+    side = torch.cuda.Stream()
+    graph = torch.cuda.CUDAGraph()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(side):
+        graph.capture_begin()
+        try:
+            rc = lib.cllm_gemm_bf16_noalloc(W.data_ptr(), X2.data_ptr(), Y.data_ptr(), 256, 256, 16, rows,
+                                            ctypes.c_void_p(side.cuda_stream))
+            Y.add_(1.0)  # the capture stays valid after the refusal
+        finally:
+            graph.capture_end()
+    assert cllm.STATUS.get(rc) == "CLLM_EUNSUPPORTED", rc
+    graph.replay()
+    torch.cuda.synchronize()
+    assert float(Y.max()) == 1.0 and float(Y.min()) == 1.0
