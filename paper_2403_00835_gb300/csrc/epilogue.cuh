@@ -40,7 +40,14 @@ struct EpiSmem {
   int bidx_all[kEpiPrepMax];
 };
 
+// Barrier of the thread's group of 4 epilogue warps: named barrier 1; in a
+// translation unit that defines CLLM_EPI_GROUPS (kernels with a second group
+// in warps 6-9), named barrier 2 for that group.
+#ifdef CLLM_EPI_GROUPS
+__device__ __forceinline__ void epi_sync() { named_bar_sync((threadIdx.x >> 5) >= 6 ? 2 : 1, 128); }
+#else
 __device__ __forceinline__ void epi_sync() { named_bar_sync(1, 128); }
+#endif
 
 // rs[t] = 1 / sqrt(sum of the per-tile sums of squares / d + eps) for the 16
 // columns t0..t0+15: 8 threads per column each sum the tiles i = part (mod 8)

@@ -25,6 +25,7 @@
 #include <float.h>
 #include <limits.h>
 
+#define CLLM_EPI_GROUPS 1  // kernels of this unit may run two epilogue groups
 #include "act.cuh"
 #include "epilogue.cuh"
 #include "gemm_roles.cuh"
@@ -45,11 +46,20 @@ using SoloCfg = TcCfg<BNMAX, BNMAX <= 32 ? 8 : (BNMAX <= 64 ? 6 : (BNMAX <= 128 
 
 constexpr int kSoloRedSlots = 2;  // split-K partial blocks staged per reduction round
 
+// Epilogue groups: at 256 token columns one accumulator fills tensor memory,
+// so the MMAs of a CTA's next unit wait for the whole epilogue of the last
+// one (16 chunks); a second group of 4 warps halves that wait.
+template <int KIND, int BNMAX>
+constexpr int solo_groups() { return BNMAX == 256 ? 2 : 1; }
+
+constexpr size_t kSoloGroupBytes = (sizeof(EpiSmem) + 15) / 16 * 16 + kSoloRedSlots * kRedSlotBytes;
+
 template <int BNMAX>
 constexpr size_t solo_smem_bytes() {
   using Cfg = SoloCfg<BNMAX>;
-  return 1024 + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES + sizeof(EpiSmem) + 16 +
-         kSoloRedSlots * kRedSlotBytes + tc_bar_bytes(Cfg::STAGES);
+  constexpr int groups = BNMAX == 256 ? 2 : 1;  // room for two groups at 256 columns
+  return 1024 + static_cast<size_t>(Cfg::STAGES) * Cfg::STAGE_BYTES + groups * kSoloGroupBytes + 16 +
+         tc_bar_bytes(Cfg::STAGES) + 16;
 }
 constexpr size_t kSmemLimit = 227 * 1024 - 256;  // minus static shared memory
 static_assert(solo_smem_bytes<32>() <= kSmemLimit && solo_smem_bytes<64>() <= kSmemLimit &&
@@ -57,17 +67,19 @@ static_assert(solo_smem_bytes<32>() <= kSmemLimit && solo_smem_bytes<64>() <= kS
               "per-GEMM kernel shared memory over the 227 KB limit");
 
 template <int KIND, int BNMAX>
-__global__ void __launch_bounds__(192, 1)
+__global__ void __launch_bounds__(64 + 128 * solo_groups<KIND, BNMAX>(), 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mA1,
                    const __grid_constant__ CUtensorMap mA2, const __grid_constant__ CUtensorMap mB,
                    const GemmArgs g, const EpiArgs e) {
   using Cfg = SoloCfg<BNMAX>;
+  constexpr int NG = solo_groups<KIND, BNMAX>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base =
       reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  EpiSmem& es = *reinterpret_cast<EpiSmem*>(base + Cfg::STAGES * Cfg::STAGE_BYTES);
-  float* red = reinterpret_cast<float*>((reinterpret_cast<uintptr_t>(&es + 1) + 15) & ~uintptr_t(15));
-  uint8_t* bars = reinterpret_cast<uint8_t*>(red) + kSoloRedSlots * kRedSlotBytes;
+  // [ring][per group: EpiSmem, staging slots][barriers][shared flag]
+  uint8_t* groups = base + Cfg::STAGES * Cfg::STAGE_BYTES;
+  uint8_t* bars = groups + (BNMAX == 256 ? 2 : 1) * kSoloGroupBytes;
+  int* jflag = reinterpret_cast<int*>(bars + tc_bar_bytes(Cfg::STAGES));
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&mA0);
@@ -75,9 +87,9 @@ __global__ void __launch_bounds__(192, 1)
     tma_prefetch_desc(&mA2);
     tma_prefetch_desc(&mB);
   }
-  TcPipe P = tc_pipe_init<Cfg>(base, bars);
-  P.red = red;
+  TcPipe P = tc_pipe_init<Cfg, NG>(base, bars);
   P.red_slots = kSoloRedSlots;
+  P.jflag = jflag;
   // Every CTA of this grid is resident (one per SM): let the next kernel in
   // the stream start its independent prologue now.
   pdl_launch_dependents();
@@ -98,9 +110,14 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     pdl_wait();
+    const int gi = (warp - 2) / 4;  // epilogue group
+    uint8_t* mine = groups + gi * kSoloGroupBytes;
+    EpiSmem& es = *reinterpret_cast<EpiSmem*>(mine);
+    TcPipe Pg = P;
+    Pg.red = reinterpret_cast<float*>(mine + (sizeof(EpiSmem) + 15) / 16 * 16);
     int acc = 0;
     uint32_t accph = 0;
-    tc_epilogue<KIND, Cfg>(P, acc, accph, g, e, c0, c1, blockIdx.x, es);
+    tc_epilogue<KIND, Cfg, NG>(Pg, acc, accph, g, e, c0, c1, blockIdx.x, es);
   }
   tc_pipe_release<Cfg>(P);
   if (threadIdx.x == 0 && *P.abort) atomicOr(g.err, DERR_TIMEOUT);
@@ -241,7 +258,7 @@ static cudaError_t launch_tc_one(const GemmMaps& m, const GemmArgs& g, const Epi
                                  cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[1];
-  fill_launch(cfg, attr, dim3(grid), dim3(192), solo_smem_bytes<BN>(), s, pdl);
+  fill_launch(cfg, attr, dim3(grid), dim3(64 + 128 * solo_groups<KIND, BN>()), solo_smem_bytes<BN>(), s, pdl);
   return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<KIND, BN>, m.a0, m.a1, m.a2, m.b, g, e);
 }
 

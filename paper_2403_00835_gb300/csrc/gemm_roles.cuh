@@ -51,6 +51,7 @@ struct TcPipe {
   // blocks of kEpiCols x kBM floats (set by the kernel after tc_pipe_init)
   float* red;
   int red_slots;
+  int* jflag;  // two epilogue groups: the split-K wait's result, shared (shared memory)
 };
 
 constexpr size_t kRedSlotBytes = sizeof(float) * kEpiCols * kBM;
@@ -60,7 +61,8 @@ __host__ __device__ constexpr size_t tc_bar_bytes(int stages) { return 8 * (2 * 
 
 // Carve the pipeline from shared memory and initialise it (all threads call).
 // `bars` must be 8-byte aligned and hold tc_bar_bytes(STAGES) bytes.
-template <class Cfg>
+// NG: epilogue groups of 4 warps (each warp releases the accumulator).
+template <class Cfg, int NG = 1>
 __device__ TcPipe tc_pipe_init(uint8_t* ring, uint8_t* bars) {
   constexpr int S = Cfg::STAGES;
   TcPipe P;
@@ -82,7 +84,7 @@ __device__ TcPipe tc_pipe_init(uint8_t* ring, uint8_t* bars) {
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&P.tfull[i], 1);
-      mbar_init(&P.tempty[i], 4);
+      mbar_init(&P.tempty[i], 4 * NG);
     }
     mbar_init(P.drain, 1);
     *P.abort = 0;
@@ -413,12 +415,22 @@ __device__ __forceinline__ void epi_publish(const EpiArgs& e, int mt, int r) {
   if (r == 0) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(e.tile_done + mt) : "memory");
 }
 
-template <int KIND, class Cfg>
+// NG = 2 (per-GEMM kernel, 256 token columns): two groups of 4 epilogue warps
+// (warps 2-5 and 6-9, each with its own named barrier, EpiSmem and staging
+// slots) take alternate 16-column chunks of each unit; a barrier over both
+// groups orders their stores before the split-K release, the ticket reset
+// and the argmax reduction.  Per column the arithmetic is unchanged.
+template <int KIND, class Cfg, int NG = 1>
 __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const GemmArgs& g,
                             const EpiArgs& e, int c0, int c1, int cta, EpiSmem& es) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int grp = warp & 3;
   const int r = grp * 32 + lane;
+  const int gi = NG > 1 ? (warp >= 6 ? 1 : 0) : 0;  // this thread's group
+  auto joint = [&]() {
+    if constexpr (NG > 1) named_bar_sync(3, 128 * NG);
+    else epi_sync();
+  };
   const bool tile_mode = g.ntiles > 1;
   if (c0 < c1) epi_prepare<KIND>(e, r, es);
   int c = c0;
@@ -427,7 +439,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     const int u = sg.unit;
     const int mt = u / g.ntiles, nt = u - mt * g.ntiles;
     EpiPre pre;
-    epi_prefetch<KIND, __nv_bfloat16>(e, mt, tile_mode ? nt * Cfg::BN : 0, r, es, pre);
+    epi_prefetch<KIND, __nv_bfloat16>(e, mt, (tile_mode ? nt * Cfg::BN : 0) + gi * kEpiCols, r, es, pre);
     if (r == 0) es.ok = mbar_wait(&P.tfull[acc], accph, P.abort) ? 1 : 0;
     epi_sync();
     const bool seg_ok = es.ok != 0;
@@ -453,7 +465,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     // the partials to its own accumulator in slot order.
     const bool owner = nc > 1 && slot == 0;
     if (!owner) {
-      for (int ch = 0; ch < nchunk; ++ch) {
+      for (int ch = gi; ch < nchunk; ch += NG) {
         float v[kEpiCols];
         tmem_ld_sum_cfg<Cfg>(taddr, ch, g.bn, v);
         if (nc == 1) {
@@ -468,17 +480,26 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
       __syncwarp();
       if (lane == 0) mbar_arrive(&P.tempty[acc]);
       if (nc > 1) {
-        epi_sync();  // every thread's partial stores precede the release
-        if (r == 0) red_release_gpu(&g.tickets[u], 1);
+        joint();  // every thread's partial stores precede the release
+        if (gi == 0 && r == 0) red_release_gpu(&g.tickets[u], 1);
         if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
       } else if (KIND == EPI_ARGMAX) {
-        epi_argmax_finish(e, r, es);
+        if constexpr (NG > 1) joint();  // both groups' partial maxima are written
+        if (gi == 0) epi_argmax_finish(e, r, es);
       }
     } else {
-      if (r == 0) es.ok = count_wait(&g.tickets[u], nc - 1, P.abort) ? 1 : 0;
-      epi_sync();
-      const bool got = es.ok != 0;
-      epi_sync();
+      bool got;
+      if constexpr (NG > 1) {
+        // one wait for both groups, so that they agree on its outcome
+        if (gi == 0 && r == 0) *P.jflag = count_wait(&g.tickets[u], nc - 1, P.abort) ? 1 : 0;
+        joint();
+        got = *P.jflag != 0;
+      } else {
+        if (r == 0) es.ok = count_wait(&g.tickets[u], nc - 1, P.abort) ? 1 : 0;
+        epi_sync();
+        got = es.ok != 0;
+        epi_sync();
+      }
       if (!got) {
         tc_fence_before();
         __syncwarp();
@@ -486,7 +507,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
         return false;
       }
       if (dbg) e.dbg[e.dbg_stride + cta] = globaltimer_ns();
-      for (int ch = 0; ch < nchunk; ++ch) {
+      for (int ch = gi; ch < nchunk; ch += NG) {
         float v[kEpiCols];
         tmem_ld_sum_cfg<Cfg>(taddr, ch, g.bn, v);
         // slots 1..nc-1: a group of up to red_slots partial blocks
@@ -505,7 +526,7 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
           }
           cp_async_commit();
           // the chunk's own epilogue inputs travel in the same round trip
-          if (ch > 0 && s0 == 1)
+          if (ch > gi && s0 == 1)
             epi_prefetch<KIND, __nv_bfloat16>(e, mt, tbase + ch * kEpiCols, r, es, pre);
           cp_async_wait_all();
           epi_sync();
@@ -521,12 +542,13 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
       }
       // (the count is reset before the tile is published: a later phase that
       // the flag opens may count on the same ticket)
-      if (r == 0) g.tickets[u] = 0;
+      if constexpr (NG > 1) joint();  // both groups are past the wait and done
+      if (gi == 0 && r == 0) g.tickets[u] = 0;
       epi_publish(e, mt, r);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&P.tempty[acc]);
-      if (KIND == EPI_ARGMAX) epi_argmax_finish(e, r, es);
+      if (KIND == EPI_ARGMAX && gi == 0) epi_argmax_finish(e, r, es);
     }
     if (dbg) e.dbg[2 * e.dbg_stride + cta] = globaltimer_ns();
     if (++acc == Cfg::NACC) {
