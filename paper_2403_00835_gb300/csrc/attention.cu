@@ -117,30 +117,39 @@ __global__ void __launch_bounds__(128) attn_chunk_simt_kernel(const AttnArgs a) 
 
 // Merge of a row's partials (per chunk range) in order; out = O / l
 // (fmaf accumulation in chunk order, as in the persistent kernel's merge).
+// One (row, head) per hd/4 threads, 4 consecutive dims per thread (vector
+// loads and stores); per element the same sums in the same order as a
+// per-element loop.
 template <typename Act>
-__global__ void attn_combine_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(128) attn_combine_kernel(const AttnArgs a) {
   pdl_launch_dependents();
   pdl_wait();
   // the tensor-core path leaves one partial per range of kAttnRange chunks,
   // the fp32 path one per chunk
   constexpr int R = std::is_same<Act, float>::value ? 1 : kAttnRange;
-  const int t = blockIdx.x / a.H, h = blockIdx.x - (blockIdx.x / a.H) * a.H;
-  if (t >= a.T) return;
+  const int tpp = a.hd / 4;  // threads per (row, head)
+  const int pair = blockIdx.x * (blockDim.x / tpp) + threadIdx.x / tpp;
+  if (pair >= a.T * a.H) return;
+  const int t = pair / a.H, h = pair - t * a.H;
+  const int d = (threadIdx.x % tpp) * 4;
   const int nch = (min(a.pos[t] / kAttnChunk + 1, a.nch_max) + R - 1) / R;
   const size_t base = (static_cast<size_t>(t) * a.H + h) * a.nch_max;
   float M = -INFINITY;
   for (int c = 0; c < nch; ++c) M = fmaxf(M, a.part_ml[base + c].x);
-  for (int d = threadIdx.x; d < a.hd; d += blockDim.x) {
-    float acc = 0.f, l = 0.f;
-    for (int c = 0; c < nch; ++c) {
-      const float2 ml = a.part_ml[base + c];
-      const float f = exp2f(ml.x - M);
-      l = fmaf(f, ml.y, l);
-      acc = fmaf(f, a.part_o[(base + c) * a.hd + d], acc);
-    }
-    st_gin(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * a.hd + h * a.hd + d, a.plane_out,
-           acc / l);
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  float l = 0.f;
+  for (int c = 0; c < nch; ++c) {
+    const float2 ml = a.part_ml[base + c];
+    const float f = exp2f(ml.x - M);
+    l = fmaf(f, ml.y, l);
+    const float4 o = *reinterpret_cast<const float4*>(a.part_o + (base + c) * a.hd + d);
+    acc.x = fmaf(f, o.x, acc.x);
+    acc.y = fmaf(f, o.y, acc.y);
+    acc.z = fmaf(f, o.z, acc.z);
+    acc.w = fmaf(f, o.w, acc.w);
   }
+  st_gin4(static_cast<Act*>(a.out), static_cast<size_t>(t) * a.H * a.hd + h * a.hd + d, a.plane_out,
+          make_float4(acc.x / l, acc.y / l, acc.z / l, acc.w / l));
 }
 
 // ---- launchers ----------------------------------------------------------------------
@@ -197,7 +206,8 @@ cudaError_t launch_attention(const AttnArgs& a, int act_bf16, int grid, cudaStre
 cudaError_t launch_attn_combine(const AttnArgs& a, int act_bf16, cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[1];
-  attn_cfg(cfg, attr, dim3(a.T * a.H), dim3(a.hd), 0, s, pdl);
+  const int per_block = 128 / (a.hd / 4);  // (row, head) pairs per 128-thread block
+  attn_cfg(cfg, attr, dim3((a.T * a.H + per_block - 1) / per_block), dim3(128), 0, s, pdl);
   if (act_bf16) return cudaLaunchKernelEx(&cfg, attn_combine_kernel<__nv_bfloat16>, a);
   return cudaLaunchKernelEx(&cfg, attn_combine_kernel<float>, a);
 }
