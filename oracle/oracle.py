@@ -18,7 +18,10 @@ Layout
                             appending fresh guesses after each commit; ``shrink``
                             follows Alg. 3 (the state shrinks by the accepted
                             count until the n-token window is fixed, then the next
-                            window starts as in Alg. 1's x <- cat(x, y*)).
+                            window starts as in Alg. 1's x <- cat(x, y*)); and
+                            ``lookahead``, the refill policy with an n-gram pool
+                            (Sec. 3.3's combination with lookahead decoding,
+                            see ``ngram_pool_step``).
         ``jacobi_step``     one iteration of the above from an explicit block.
         ``jacobi_vanilla``  Eq. 3 iterated without any cache until
                             y^(k) = y^(k-1) (Sec. 3.1), used only as a pin.
@@ -32,6 +35,16 @@ Readings of the paper this oracle takes:
   * The next head is P[a-1]; refill keeps P[a-1:] and appends a-1 fresh guesses.
   * Argmax ties go to the lowest token id; gap = top1 - top2 of the raw logits
     (duplicates allowed, so gap may be 0).
+  * Lookahead combination (Sec. 3.3 gives one sentence: n-grams generated
+    in previous Jacobi iterations are collected as candidates and verified in
+    the next iteration).  Reading: each iteration's predictions P are an
+    n-gram source -- for every k with k + N - 1 < n, key P[k] and value
+    P[k+1..k+N-1] (N = n-gram size), later k replacing earlier ones under the
+    same key.  Before the iteration's n-grams enter the pool, the next block
+    (the refill block) takes the pool's value for its head P[a-1], if there is
+    one, in slots 1..N-1; the next iteration's acceptance verifies it.  One
+    candidate per iteration, inside the Jacobi block: no separate lookahead
+    window and no parallel verification branch.
   * Guesses ("random tokens", Alg. 3) are drawn from a counter-based
     splitmix64 stream (Vigna), keyed by (seed, sequence b, iteration, slot):
     uniform over the vocabulary, or uniform over the prompt's tokens.
@@ -352,9 +365,27 @@ def ar_decode(model: OracleModel, prompt: Sequence[int], max_new: int, eos_id: i
     return DecodeResult(out, passes, [1] * len(out), gaps[:len(out)])
 
 
+def ngram_pool_step(pool: dict, pred: Sequence[int], a: int, block: Sequence[int], ngram: int) -> list:
+    """The lookahead policy's step (reading of Sec. 3.3 in the module header):
+    the refill ``block`` takes the pool's (ngram - 1)-token continuation of
+    its head pred[a-1] in slots 1.., then this iteration's n-grams of ``pred``
+    enter ``pool`` (key pred[k], value pred[k+1 .. k+ngram-1], k ascending).
+    Returns the next block; ``pool`` is updated in place."""
+    W = ngram - 1
+    out = list(block)
+    cand = pool.get(pred[a - 1])
+    if cand is not None:
+        w = min(W, len(out) - 1)
+        out[1:1 + w] = cand[:w]
+    for k in range(len(pred) - W):
+        pool[pred[k]] = list(pred[k + 1:k + 1 + W])
+    return out
+
+
 def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: int, seed: int,
                   b: int = 0, mode: str = "refill", guess_init: str = "uniform",
-                  eos_id: int = -1, record: bool = False, keep_steps: bool = False) -> DecodeResult:
+                  eos_id: int = -1, record: bool = False, keep_steps: bool = False,
+                  ngram: int = 4) -> DecodeResult:
     """Jacobi decoding with KV cache (Alg. 3) of one sequence ``b``.
 
     Each iteration forwards the current block over the committed cache,
@@ -364,7 +395,9 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
     guesses, ``shrink`` lets it shrink until the window is fixed.
     ``record`` keeps the block of every iteration and ``keep_steps`` every
     iteration's StepResult with its logits (recorded only, never used)."""
-    assert mode in ("refill", "shrink") and n >= 1 and max_new >= 1
+    assert mode in ("refill", "shrink", "lookahead") and n >= 1 and max_new >= 1
+    assert mode != "lookahead" or ngram >= 2
+    pool: dict = {}
     V = model.arch.vocab
     src = list(prompt) if guess_init == "prompt" else None
 
@@ -398,8 +431,10 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
         if stop or len(res.tokens) >= max_new:
             break
         it = res.iterations
-        if mode == "refill":
+        if mode in ("refill", "lookahead"):
             block = st.pred[a - 1:] + [g(it, i) for i in range(m - a + 1, m)]
+            if mode == "lookahead":
+                block = ngram_pool_step(pool, st.pred, a, block, ngram)
         elif a == m:
             block = [st.pred[m - 1]] + [g(it, i) for i in range(1, n)]
         else:

@@ -167,3 +167,43 @@ def test_brute_force_micro_model(micro):
         for mode in ("refill", "shrink"):
             assert orc.jacobi_decode(m, prompt, n, 12, seed=seed, mode=mode).tokens == \
                 orc.ar_decode(m, prompt, 12).tokens
+
+
+# ---- the lookahead combination (Sec. 3.3): n-gram pool feeding the refill block
+
+def test_ngram_pool_step_worked_example():
+    """Hand-worked step of the pool rule: predictions [5, 6, 7, 8, 9], two
+    tokens accepted, trigrams (two-token values).  The head 6 has the pool
+    continuation [1, 2], which replaces refill slots 1-2; the iteration's
+    trigrams keyed 5, 6, 7 then enter the pool (6's value replaced)."""
+    pool = {6: [1, 2]}
+    out = orc.ngram_pool_step(pool, [5, 6, 7, 8, 9], 2, [6, 7, 8, 9, 42], 3)
+    assert out == [6, 1, 2, 9, 42]
+    assert pool == {5: [6, 7], 6: [7, 8], 7: [8, 9]}
+
+
+def test_ngram_pool_step_edges():
+    # no entry for the head: the refill block unchanged
+    pool = {}
+    assert orc.ngram_pool_step(pool, [3, 3, 4, 3, 5], 1, [3, 3, 4, 3, 5], 2) == [3, 3, 4, 3, 5]
+    # the same key several times in one iteration: the last n-gram wins
+    assert pool == {3: [5], 4: [3]}
+    # a candidate longer than the block is cut at the block's end; a block
+    # shorter than the n-gram adds nothing to the pool
+    pool = {7: [1, 2, 3, 4, 5]}
+    assert orc.ngram_pool_step(pool, [7, 0, 0], 1, [7, 9, 9], 6) == [7, 1, 2]
+    assert pool == {7: [1, 2, 3, 4, 5]}
+
+
+@pytest.mark.parametrize("n,ngram,seed", [(8, 3, 2), (8, 5, 3), (16, 4, 4), (4, 2, 5)])
+def test_lookahead_decode_equals_ar(tiny, n, ngram, seed):
+    """Whatever the pool proposes, a token is committed only when the step
+    verifies it, so the decode is the greedy AR output (Sec. 3.1)."""
+    cfg, m = tiny
+    for pl in (32, 9):
+        prompt = syn.make_prompts(cfg.vocab, [pl], seed=seed)[0]
+        ar = orc.ar_decode(m, prompt, 40)
+        jr = orc.jacobi_decode(m, prompt, n, 40, seed=seed, mode="lookahead", ngram=ngram)
+        assert jr.tokens == ar.tokens
+        assert all(a >= 1 for a in jr.accepted)
+        assert sum(jr.accepted) == 40
