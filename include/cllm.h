@@ -54,6 +54,13 @@ extern "C" {
 #define CLLM_BLOCK_REFILL 0       /* block stays n wide: fresh guesses after commits */
 #define CLLM_BLOCK_SHRINK 1       /* Alg. 3: the window narrows by the accepted tokens
                                      until it is fixed, then a fresh n-wide block */
+#define CLLM_BLOCK_LOOKAHEAD 2    /* refill, with an n-gram pool (Sec. 3.3's combination
+                                     with lookahead decoding): each iteration's
+                                     predictions P give n-grams (key P[k], value
+                                     P[k+1..k+ngram-1]); the next block takes the
+                                     pooled continuation of its head in slots
+                                     1..ngram-1 (from earlier iterations' n-grams),
+                                     and the step verifies it */
 
 /*
  * Model shape and capacity.  The decoder is the pre-norm LLaMA layer:
@@ -93,11 +100,15 @@ typedef struct {
   uint64_t seed;   /* key of the counter-based guess generator                    */
   int eos_id;      /* -1: off.  Else a sequence stops after committing this token   */
   int guess_init;  /* CLLM_GUESS_UNIFORM | CLLM_GUESS_FROM_PROMPT                  */
-  int block_mode;  /* CLLM_BLOCK_REFILL | CLLM_BLOCK_SHRINK                       */
+  int block_mode;  /* CLLM_BLOCK_REFILL | CLLM_BLOCK_SHRINK | CLLM_BLOCK_LOOKAHEAD  */
   int record_cap;  /* > 0: record the first record_cap blocks of every sequence
                       (the Jacobi trajectory), read with cllm_decode_read_trajectory */
   int stats;       /* 1: keep the acceptance statistics on the device, read with
                       cllm_decode_read_stats; 0: off                           */
+  int ngram;       /* CLLM_BLOCK_LOOKAHEAD: n-gram size, 2..16 (the pool keeps
+                      ngram - 1 tokens per key token, one pool per sequence,
+                      batch * vocab * (ngram - 1) ints of device memory); other
+                      modes: ignored                                             */
 } cllm_decode_opts;
 
 /* Acceptance statistics of a decode (Sec. 3.3, Table 3), summed over the

@@ -22,6 +22,7 @@ CLLM_F32, CLLM_BF16 = 0, 1
 CLLM_GUESS_UNIFORM, CLLM_GUESS_FROM_PROMPT = 0, 1
 CLLM_BLOCK_REFILL = 0
 CLLM_BLOCK_SHRINK = 1
+CLLM_BLOCK_LOOKAHEAD = 2
 
 # Every function declared in include/cllm.h.
 EXPORTS = ("cllm_create", "cllm_destroy", "cllm_prefill", "cllm_jacobi_step", "cllm_jacobi_decode",
@@ -62,7 +63,8 @@ class Weights(ctypes.Structure):
 
 class DecodeOpts(ctypes.Structure):
     _fields_ = [("seed", ctypes.c_uint64), ("eos_id", ctypes.c_int), ("guess_init", ctypes.c_int),
-                ("block_mode", ctypes.c_int), ("record_cap", ctypes.c_int), ("stats", ctypes.c_int)]
+                ("block_mode", ctypes.c_int), ("record_cap", ctypes.c_int), ("stats", ctypes.c_int),
+                ("ngram", ctypes.c_int)]
 
 
 class AcceptStats(ctypes.Structure):
@@ -238,7 +240,7 @@ class Engine:
 
     def jacobi_decode(self, prompts, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
                       guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL,
-                      record_cap: int = 0, stats: bool = False):
+                      record_cap: int = 0, stats: bool = False, ngram: int = 4):
         """Tokens [B][max_new] and iterations [B]; with record_cap > 0 also the
         trajectory [record_cap][B][n] (-1 outside the window).  With stats the
         device keeps the acceptance statistics (read with decode_read_stats)."""
@@ -246,7 +248,7 @@ class Engine:
         B = len(prompts)
         out = np.zeros((B, max_new), dtype=np.int32)
         its = np.zeros(B, dtype=np.int32)
-        o = DecodeOpts(seed, eos_id, guess_init, block_mode, record_cap, 1 if stats else 0)
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, record_cap, 1 if stats else 0, ngram)
         _check(self._lib.cllm_jacobi_decode(self._h, B, _ip(toks), _ip(lens), n, max_new,
                                             ctypes.byref(o), _ip(out), _ip(its)), "cllm_jacobi_decode")
         self.B = B
@@ -269,8 +271,8 @@ class Engine:
 
     def decode_begin(self, n: int, max_new: int, seed: int = 0, eos_id: int = -1,
                      guess_init: int = CLLM_GUESS_UNIFORM, block_mode: int = CLLM_BLOCK_REFILL,
-                     stats: bool = False):
-        o = DecodeOpts(seed, eos_id, guess_init, block_mode, 0, 1 if stats else 0)
+                     stats: bool = False, ngram: int = 4):
+        o = DecodeOpts(seed, eos_id, guess_init, block_mode, 0, 1 if stats else 0, ngram)
         _check(self._lib.cllm_decode_begin(self._h, n, max_new, ctypes.byref(o)), "cllm_decode_begin")
         self._dec_max_new = max_new
         self._dec_n = n

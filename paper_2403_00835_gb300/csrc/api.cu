@@ -162,6 +162,8 @@ struct cllm_ctx {
       *win_cnt = nullptr;
   int* traj = nullptr;  // recorded trajectory [traj_cap][B][n]
   size_t traj_alloc = 0;
+  int* pool = nullptr;  // lookahead policy's n-gram pools [B][V][ngram - 1]
+  size_t pool_alloc = 0;
   int traj_cap = 0;
   int* status_host = nullptr;  // pinned: slots of 4 ints {active, committed, device error, -}
   cudaEvent_t iter_ev[2] = {nullptr, nullptr};
@@ -545,6 +547,10 @@ AcceptArgs make_accept(cllm_ctx* c, int B, int n, bool decode) {
   a.status = c->status;
   a.shrink = (decode && c->dec_opts.block_mode == CLLM_BLOCK_SHRINK) ? 1 : 0;
   a.width = c->width;
+  if (decode && c->dec_opts.block_mode == CLLM_BLOCK_LOOKAHEAD) {
+    a.pool = c->pool;
+    a.pool_w = c->dec_opts.ngram - 1;
+  }
   a.traj = (decode && c->traj_cap > 0) ? c->traj : nullptr;
   a.traj_cap = decode ? c->traj_cap : 0;
   if (decode && c->dec_opts.stats) {
@@ -813,7 +819,8 @@ int get_graph(cllm_ctx* c, int mode, int n, cllm_ctx::GraphEntry** out) {
                                                     (c->traj_cap << 4))
                                                  : 0,
                              (c->profiling ? 1 : 0) | (mode == MODE_STEP && c->step_logits ? 2 : 0) |
-                                 (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0),
+                                 (mode == MODE_DECODE && c->dec_opts.stats ? 4 : 0) |
+                                 (mode == MODE_DECODE ? (c->dec_opts.ngram << 3) : 0),
                              c->persistent ? 1 : 0,
                              (c->park_slots * 4096 + c->l2_pairs) * 2 + (c->dataflow ? 1 : 0));
   auto it = c->graphs.find(key);
@@ -1472,7 +1479,11 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
   o.block_mode = CLLM_BLOCK_REFILL;
   if (opts) o = *opts;
   if (o.guess_init != CLLM_GUESS_UNIFORM && o.guess_init != CLLM_GUESS_FROM_PROMPT) return CLLM_EINVAL;
-  if (o.block_mode != CLLM_BLOCK_REFILL && o.block_mode != CLLM_BLOCK_SHRINK) return CLLM_EINVAL;
+  if (o.block_mode != CLLM_BLOCK_REFILL && o.block_mode != CLLM_BLOCK_SHRINK &&
+      o.block_mode != CLLM_BLOCK_LOOKAHEAD)
+    return CLLM_EINVAL;
+  if (o.block_mode == CLLM_BLOCK_LOOKAHEAD && (o.ngram < 2 || o.ngram > 16)) return CLLM_EINVAL;
+  if (o.block_mode != CLLM_BLOCK_LOOKAHEAD) o.ngram = 0;
   if (o.record_cap < 0 || o.record_cap > (1 << 20)) return CLLM_EINVAL;
   if (o.stats != 0 && o.stats != 1) return CLLM_EINVAL;
   if (o.eos_id >= c->V) return CLLM_EINVAL;
@@ -1496,6 +1507,14 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
     c->out_cap = need;
     stale = true;
   }
+  const size_t pool_need = o.ngram > 0 ? static_cast<size_t>(c->B) * c->V * (o.ngram - 1) : 0;
+  if (pool_need > c->pool_alloc) {
+    int* p = nullptr;
+    if (!dev_alloc(c, &p, pool_need * 4)) return CLLM_ENOMEM;
+    c->pool = p;
+    c->pool_alloc = pool_need;
+    stale = true;
+  }
   if (stale) {
     // graphs captured against the old output buffer are stale
     for (auto& kv : c->graphs) {
@@ -1510,6 +1529,9 @@ extern "C" int cllm_decode_begin(cllm_ctx* c, int n, int max_new, const cllm_dec
   c->dec_opts = o;
   c->traj_cap = o.record_cap;
   if (traj_need > 0 && cudaMemsetAsync(c->traj, 0xff, traj_need * 4, c->stream) != cudaSuccess)
+    return CLLM_ECUDA;
+  // an empty pool: every entry -1
+  if (pool_need > 0 && cudaMemsetAsync(c->pool, 0xff, pool_need * 4, c->stream) != cudaSuccess)
     return CLLM_ECUDA;
   if (cudaMemcpyAsync(c->head, c->head0, c->B * 4, cudaMemcpyDeviceToDevice, c->stream) !=
       cudaSuccess)

@@ -168,6 +168,11 @@ struct AcceptArgs {
   // narrows by the accepted count until it is fixed, then a fresh n-wide block)
   int shrink;
   int* width;  // [B] current block width (shrink)
+  // lookahead policy (refill with an n-gram pool; null: off): pool[b][tok]
+  // holds the pool_w tokens that followed tok in the latest n-gram of
+  // sequence b's predictions, pool[b][tok][0] = -1 when there is none
+  int* pool;
+  int pool_w;
   // optional trajectory: traj[it][b][k] = the block of sequence b at its
   // iteration it (slot k < width, -1 beyond), for it < traj_cap
   int* traj;

@@ -164,6 +164,21 @@ __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, 
         const int keep = n - acc + 1;
         const int step = a.iters[b];
         for (int k = 0; k < n; ++k) y[k] = (k < keep) ? P[acc - 1 + k] : draw_guess(a, b, step, k);
+        if (a.pool != nullptr) {
+          // lookahead (Sec. 3.3): the pooled continuation of the new head,
+          // from earlier iterations, fills slots 1..; then this iteration's
+          // n-grams (key P[k], value P[k+1..k+pool_w], k ascending) enter
+          int* pb = a.pool + static_cast<size_t>(b) * a.V * a.pool_w;
+          const int* cand = pb + static_cast<size_t>(P[acc - 1]) * a.pool_w;
+          if (cand[0] >= 0) {
+            const int w = min(a.pool_w, n - 1);
+            for (int j = 0; j < w; ++j) y[1 + j] = cand[j];
+          }
+          for (int k = 0; k + a.pool_w < n; ++k) {
+            int* dst = pb + static_cast<size_t>(P[k]) * a.pool_w;
+            for (int j = 0; j < a.pool_w; ++j) dst[j] = P[k + 1 + j];
+          }
+        }
       } else if (a.decode) {
         const int step = a.iters[b];
         if (acc == w) {
