@@ -164,6 +164,8 @@ struct cllm_ctx {
   size_t traj_alloc = 0;
   int* pool = nullptr;  // lookahead policy's n-gram pools [B][V][ngram - 1]
   size_t pool_alloc = 0;
+  AttnMaps attn_maps{};     // bf16 engine: tensor maps of the attention tiles
+  bool attn_maps_ok = false;
   int traj_cap = 0;
   int* status_host = nullptr;  // pinned: slots of 4 ints {active, committed, device error, -}
   cudaEvent_t iter_ev[2] = {nullptr, nullptr};
@@ -458,9 +460,13 @@ cudaError_t record_forward(cllm_ctx* c, cudaStream_t s, const FwdSpec& f, bool p
     // (a3) block attention, split over position-anchored key chunks
     aa.k_cache = kl;
     aa.v_cache = vl;
-    if ((err = after_launch(c, s, "attention", launch_attention(aa, ab, f.attn_grid, s, pdl))) !=
-        cudaSuccess)
-      return err;
+    {
+      const int kv_row0 = static_cast<int>(static_cast<size_t>(l) * c->layer_kv_elems / c->hd);
+      const cudaError_t la = c->attn_maps_ok
+                                 ? launch_attention_tma(aa, c->attn_maps, kv_row0, f.attn_grid, s, pdl)
+                                 : launch_attention(aa, ab, f.attn_grid, s, pdl);
+      if ((err = after_launch(c, s, "attention", la)) != cudaSuccess) return err;
+    }
     if ((err = after_launch(c, s, "attn_combine", launch_attn_combine(aa, ab, s, pdl))) !=
         cudaSuccess)
       return err;
@@ -1199,6 +1205,15 @@ extern "C" int cllm_create(const cllm_arch* arch, const cllm_weights* w, void* c
     if (!ok) {
       rc = CLLM_ENOMEM;
       break;
+    }
+    // tensor maps of the per-GEMM attention's TMA tiles (the cache rows of
+    // all layers must be addressable with 32-bit coordinates)
+    if (c->bf16 && (c->hd == 64 || c->hd == 128)) {
+      const uint64_t kv_rows = static_cast<uint64_t>(a.n_layers) * c->layer_kv_elems / c->hd;
+      c->attn_maps_ok = kv_rows + kAttnChunk < (1ull << 31) &&
+                        make_map(&c->attn_maps.k, c->kc, c->hd, kv_rows, kAttnChunk) &&
+                        make_map(&c->attn_maps.v, c->vc, c->hd, kv_rows, kAttnChunk) &&
+                        make_map(&c->attn_maps.q, c->q, c->dq, static_cast<uint64_t>(c->Tcap), kQTile);
     }
     // RoPE table (cos, sin) of pos * theta^(-2i/hd), evaluated in double
     {

@@ -53,6 +53,32 @@ __global__ void __launch_bounds__(128) attn_chunk_mma_kernel(const AttnArgs a) {
   }
 }
 
+// The same items with Q, K and V tiles loaded by TMA from tensor maps (the
+// persistent kernel's tile path; per-thread cp.async copies reach only a
+// fraction of an SM's load bandwidth).
+template <int HD>
+constexpr size_t attn_tma_smem_bytes() {
+  return 1024 + (sizeof(AttnTileSmemTma<HD>) + 15) / 16 * 16 + sizeof(int) * (kMaxQTilesSmem + 1);
+}
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_chunk_tma_kernel(const __grid_constant__ AttnMaps m,
+                                                             const AttnArgs a, int kv_row0) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base =
+      reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  AttnTileSmemTma<HD>& t = *reinterpret_cast<AttnTileSmemTma<HD>*>(base);
+  int* pre = reinterpret_cast<int*>(base + (sizeof(AttnTileSmemTma<HD>) + 15) / 16 * 16);
+  pdl_launch_dependents();
+  pdl_wait();
+  const int total = attn_item_prefix(a, pre, threadIdx.x, CtaSync{});
+  const AttnTma tma{&m.k, &m.v, &m.q, kv_row0};
+  for (int item = blockIdx.x; item < total; item += gridDim.x) {
+    int qi, h;
+    attn_mma_item<HD>(a, item, pre, t, threadIdx.x, CtaSync{}, qi, h, GlobalMeta{a}, false, &tma);
+  }
+}
+
 // fp32 (and generic) path: one warp per row, online softmax over the chunk.
 template <typename Act, int HD>
 __global__ void __launch_bounds__(128) attn_chunk_simt_kernel(const AttnArgs a) {
@@ -170,9 +196,16 @@ cudaError_t attention_set_attributes() {
                              static_cast<int>(cudaSharedmemCarveoutMaxShared));
     if (e != cudaSuccess) return e;
   }
-  return cudaFuncSetAttribute(attn_chunk_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              static_cast<int>(sizeof(AttnSmemF16<128>)));
+  e = cudaFuncSetAttribute(attn_chunk_mma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(sizeof(AttnSmemF16<128>)));
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(attn_chunk_tma_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(attn_tma_smem_bytes<64>()));
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_chunk_tma_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(attn_tma_smem_bytes<128>()));
 }
+
 
 static void attn_cfg(cudaLaunchConfig_t& cfg, cudaLaunchAttribute* attr, dim3 grid, dim3 block,
                      size_t smem, cudaStream_t s, bool pdl) {
@@ -200,6 +233,22 @@ cudaError_t launch_attention(const AttnArgs& a, int act_bf16, int grid, cudaStre
   attn_cfg(cfg, attr, dim3(grid), dim3(128), 0, s, pdl);
   if (a.hd == 64) return cudaLaunchKernelEx(&cfg, attn_chunk_simt_kernel<float, 64>, a);
   if (a.hd == 128) return cudaLaunchKernelEx(&cfg, attn_chunk_simt_kernel<float, 128>, a);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_attention_tma(const AttnArgs& a, const AttnMaps& m, int kv_row0, int grid,
+                                 cudaStream_t s, bool pdl) {
+  if (a.n_qtiles > kMaxQTilesSmem) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  if (a.hd == 64) {
+    attn_cfg(cfg, attr, dim3(grid), dim3(128), attn_tma_smem_bytes<64>(), s, pdl);
+    return cudaLaunchKernelEx(&cfg, attn_chunk_tma_kernel<64>, m, a, kv_row0);
+  }
+  if (a.hd == 128) {
+    attn_cfg(cfg, attr, dim3(grid), dim3(128), attn_tma_smem_bytes<128>(), s, pdl);
+    return cudaLaunchKernelEx(&cfg, attn_chunk_tma_kernel<128>, m, a, kv_row0);
+  }
   return cudaErrorInvalidValue;
 }
 

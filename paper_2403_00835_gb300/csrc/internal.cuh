@@ -277,6 +277,13 @@ struct GemmMaps {
   CUtensorMap a0, a1, a2, b;
 };
 
+// Tensor maps of the attention tiles: the K and V caches of all layers as rows
+// of hd values (128-row boxes) and Q (16-row boxes), 64-column halves with the
+// 128-byte swizzle.
+struct AttnMaps {
+  CUtensorMap k, v, q;
+};
+
 inline int ceil_div(int a, int b) { return (a + b - 1) / b; }
 inline int round_up(int a, int b) { return ceil_div(a, b) * b; }
 
@@ -294,6 +301,10 @@ cudaError_t launch_gemm_tc(int kind, int bn_max, const GemmMaps& maps, const Gem
 cudaError_t launch_gemm_simt(int kind, const GemmArgs& g, const EpiArgs& e, cudaStream_t s,
                              bool pdl);
 cudaError_t launch_attention(const AttnArgs& a, int act_bf16, int grid, cudaStream_t s, bool pdl);
+// bf16 engine with tensor maps: Q, K and V tiles by TMA (kv_row0: the layer's
+// first cache row in the maps)
+cudaError_t launch_attention_tma(const AttnArgs& a, const AttnMaps& m, int kv_row0, int grid,
+                                 cudaStream_t s, bool pdl);
 cudaError_t launch_attn_combine(const AttnArgs& a, int act_bf16, cudaStream_t s, bool pdl);
 cudaError_t launch_accept(const AcceptArgs& a, cudaStream_t s, bool pdl);
 cudaError_t launch_decode_init(const AcceptArgs& a, cudaStream_t s);
