@@ -168,13 +168,19 @@ __device__ void accept_body(const AcceptArgs& a, int b, int* s_act, int* s_com, 
           // lookahead (Sec. 3.3): the pooled continuation of the new head,
           // from earlier iterations, fills slots 1..; then this iteration's
           // n-grams (key P[k], value P[k+1..k+pool_w], k ascending) enter
+          // (a prediction outside the vocabulary -- only after a device
+          // error -- is never used as a key)
           int* pb = a.pool + static_cast<size_t>(b) * a.V * a.pool_w;
-          const int* cand = pb + static_cast<size_t>(P[acc - 1]) * a.pool_w;
-          if (cand[0] >= 0) {
-            const int w = min(a.pool_w, n - 1);
-            for (int j = 0; j < w; ++j) y[1 + j] = cand[j];
+          const int h = P[acc - 1];
+          if (static_cast<unsigned>(h) < static_cast<unsigned>(a.V)) {
+            const int* cand = pb + static_cast<size_t>(h) * a.pool_w;
+            if (cand[0] >= 0) {
+              const int w = min(a.pool_w, n - 1);
+              for (int j = 0; j < w; ++j) y[1 + j] = cand[j];
+            }
           }
           for (int k = 0; k + a.pool_w < n; ++k) {
+            if (static_cast<unsigned>(P[k]) >= static_cast<unsigned>(a.V)) continue;
             int* dst = pb + static_cast<size_t>(P[k]) * a.pool_w;
             for (int j = 0; j < a.pool_w; ++j) dst[j] = P[k + 1 + j];
           }
