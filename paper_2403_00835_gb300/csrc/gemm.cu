@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(64 + 128 * solo_groups<KIND, BNMAX>(), 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* base =
       reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  // [ring][per group: EpiSmem, staging slots][barriers][shared flag]
+  // [ring][per group: EpiSmem, staging slots][barriers][shared flags, 16 bytes]
   uint8_t* groups = base + Cfg::STAGES * Cfg::STAGE_BYTES;
   uint8_t* bars = groups + (BNMAX == 256 ? 2 : 1) * kSoloGroupBytes;
   int* jflag = reinterpret_cast<int*>(bars + tc_bar_bytes(Cfg::STAGES));

@@ -51,7 +51,7 @@ struct TcPipe {
   // blocks of kEpiCols x kBM floats (set by the kernel after tc_pipe_init)
   float* red;
   int red_slots;
-  int* jflag;  // two epilogue groups: the split-K wait's result, shared (shared memory)
+  int* jflag;  // two epilogue groups, shared memory: [0] the split-K wait's result, [1] the accumulator wait's
 };
 
 constexpr size_t kRedSlotBytes = sizeof(float) * kEpiCols * kBM;
@@ -440,10 +440,20 @@ __device__ bool tc_epilogue(const TcPipe& P, int& acc, uint32_t& accph, const Ge
     const int mt = u / g.ntiles, nt = u - mt * g.ntiles;
     EpiPre pre;
     epi_prefetch<KIND, __nv_bfloat16>(e, mt, (tile_mode ? nt * Cfg::BN : 0) + gi * kEpiCols, r, es, pre);
-    if (r == 0) es.ok = mbar_wait(&P.tfull[acc], accph, P.abort) ? 1 : 0;
-    epi_sync();
-    const bool seg_ok = es.ok != 0;
-    epi_sync();
+    bool seg_ok;
+    if constexpr (NG > 1) {
+      // one wait for both groups: a group that returned alone would leave the
+      // other at the joint barrier, which has no time limit
+      if (gi == 0 && r == 0) P.jflag[1] = mbar_wait(&P.tfull[acc], accph, P.abort) ? 1 : 0;
+      joint();
+      seg_ok = P.jflag[1] != 0;
+      joint();  // read by all before the next unit's wait writes it again
+    } else {
+      if (r == 0) es.ok = mbar_wait(&P.tfull[acc], accph, P.abort) ? 1 : 0;
+      epi_sync();
+      seg_ok = es.ok != 0;
+      epi_sync();
+    }
     if (!seg_ok) return false;
     const bool dbg = e.dbg != nullptr && r == 0 && c >= c1;  // last segment
     if (dbg) e.dbg[cta] = globaltimer_ns();
