@@ -21,7 +21,10 @@ Layout
                             window starts as in Alg. 1's x <- cat(x, y*)); and
                             ``lookahead``, the refill policy with an n-gram pool
                             (Sec. 3.3's combination with lookahead decoding,
-                            see ``ngram_pool_step``).
+                            see ``ngram_pool_step``); ``verify``, the refill
+                            policy with a verification branch of several
+                            pooled n-grams (``ngram_pool_push``,
+                            ``verify_candidates``).
         ``jacobi_step``     one iteration of the above from an explicit block.
         ``jacobi_vanilla``  Eq. 3 iterated without any cache until
                             y^(k) = y^(k-1) (Sec. 3.1), used only as a pin.
@@ -45,6 +48,17 @@ Readings of the paper this oracle takes:
     one, in slots 1..N-1; the next iteration's acceptance verifies it.  One
     candidate per iteration, inside the Jacobi block: no separate lookahead
     window and no parallel verification branch.
+  * The same combination with a verification branch (``verify``): the same
+    n-gram source, but a key keeps up to G distinct values, most recent first.
+    Each iteration verifies, beside the Jacobi block, every pooled value c of
+    the block's head h, each as its own causal sequence [h, c] over the
+    committed cache (in one batched pass this is a mask under which a
+    candidate's rows see the cache, h and their own earlier rows only).  The
+    longest accepted run is committed (the block wins ties, then the most
+    recent n-gram) with its own K/V; the next head is that run's prediction
+    after its last accepted row, followed by the block's predictions for the
+    positions after it and fresh guesses (the refill block when the block
+    won).  The iteration's n-grams enter the pool after the verification.
   * Guesses ("random tokens", Alg. 3) are drawn from a counter-based
     splitmix64 stream (Vigna), keyed by (seed, sequence b, iteration, slot):
     uniform over the vocabulary, or uniform over the prompt's tokens.
@@ -343,6 +357,8 @@ class DecodeResult:
     min_gap_all: list = field(default_factory=list)  # per iteration: min gap over every row of the block
     trajectory: list = field(default_factory=list)  # blocks fed to each iteration
     steps: list = field(default_factory=list)  # StepResult of each iteration (keep_steps)
+    branch: list = field(default_factory=list)  # verify: per iteration -1 (the block) or the candidate committed
+    candidates: list = field(default_factory=list)  # verify (record): the n-grams verified per iteration
 
 
 def ar_decode(model: OracleModel, prompt: Sequence[int], max_new: int, eos_id: int = -1) -> DecodeResult:
@@ -382,10 +398,49 @@ def ngram_pool_step(pool: dict, pred: Sequence[int], a: int, block: Sequence[int
     return out
 
 
+def ngram_pool_push(pool: dict, pred: Sequence[int], ngram: int, ncand: int) -> None:
+    """The verification branch's pool (reading of Sec. 3.3 in the module
+    header): this iteration's n-grams of ``pred`` (key pred[k], value
+    pred[k+1 .. k+ngram-1], k ascending) enter ``pool``, where a key keeps at
+    most ``ncand`` distinct values, the most recently entered first (an
+    n-gram already held moves to the front)."""
+    W = ngram - 1
+    for k in range(len(pred) - W):
+        v = tuple(pred[k + 1:k + 1 + W])
+        held = pool.setdefault(pred[k], [])
+        if v in held:
+            held.remove(v)
+        held.insert(0, v)
+        del held[ncand:]
+
+
+def verify_candidates(sess: OracleSession, head: int, cands: Sequence[Sequence[int]], L: int) -> list:
+    """The verification branch of one iteration: candidate c is checked by
+    the causal forward of [head, c] over the committed cache of length L,
+    alone (no row of another candidate or of the Jacobi block is visible to
+    it).  Its accepted count is defined as the Jacobi block's: 1 + the number
+    of leading j with c[j] equal to the prediction of the row before it.
+    Returns (accepted, predictions, gaps) per candidate; the cache past L
+    holds the last candidate's K/V afterwards."""
+    out = []
+    for c in cands:
+        toks = [head] + list(c)
+        q, gaps = [], []
+        for r in sess.forward(toks, L):
+            t, gp = argmax_top2(r)
+            q.append(t)
+            gaps.append(gp)
+        a = 1
+        while a < len(toks) and toks[a] == q[a - 1]:
+            a += 1
+        out.append((a, q, gaps))
+    return out
+
+
 def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: int, seed: int,
                   b: int = 0, mode: str = "refill", guess_init: str = "uniform",
                   eos_id: int = -1, record: bool = False, keep_steps: bool = False,
-                  ngram: int = 4) -> DecodeResult:
+                  ngram: int = 4, ncand: int = 4) -> DecodeResult:
     """Jacobi decoding with KV cache (Alg. 3) of one sequence ``b``.
 
     Each iteration forwards the current block over the committed cache,
@@ -393,10 +448,16 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
     forms the next block from the remaining predictions (Alg. 3's
     z_next <- z_next[>= i*]); ``refill`` tops the block up to n with fresh
     guesses, ``shrink`` lets it shrink until the window is fixed.
-    ``record`` keeps the block of every iteration and ``keep_steps`` every
-    iteration's StepResult with its logits (recorded only, never used)."""
-    assert mode in ("refill", "shrink", "lookahead") and n >= 1 and max_new >= 1
-    assert mode != "lookahead" or ngram >= 2
+    ``verify`` adds the verification branch (module header): up to ``ncand``
+    pooled n-grams following the head are verified beside the block, and the
+    longest accepted run is committed (the block wins ties, then the most
+    recent n-gram).
+    ``record`` keeps the block of every iteration (and, for ``verify``, the
+    candidates verified) and ``keep_steps`` every iteration's StepResult with
+    its logits (recorded only, never used)."""
+    assert mode in ("refill", "shrink", "lookahead", "verify") and n >= 1 and max_new >= 1
+    assert mode not in ("lookahead", "verify") or ngram >= 2
+    assert mode != "verify" or ncand >= 1
     pool: dict = {}
     V = model.arch.vocab
     src = list(prompt) if guess_init == "prompt" else None
@@ -417,15 +478,31 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
             res.steps.append(st)
         m = len(block)
         a = st.accepted
+        # the committed run: the block's, or a verified candidate's
+        toks, pred, gaps, gaps_all = block, st.pred, st.gap, list(st.gap)
+        if mode == "verify":
+            cands = list(pool.get(block[0], []))  # from earlier iterations only
+            if record:
+                res.candidates.append([list(c) for c in cands])
+            best = -1
+            for i, (ac, q, gq) in enumerate(verify_candidates(sess, block[0], cands, L)):
+                gaps_all += gq
+                if ac > a:
+                    a, toks, pred, gaps, best = ac, [block[0]] + list(cands[i]), q, gq, i
+            res.branch.append(best)
         stop = False
-        if eos_id >= 0 and eos_id in block[:a]:
-            a = block.index(eos_id) + 1
+        if eos_id >= 0 and eos_id in toks[:a]:
+            a = toks.index(eos_id) + 1
             stop = True
         a = min(a, max_new - len(res.tokens))
-        res.tokens += block[:a]
+        res.tokens += toks[:a]
         res.accepted.append(a)
-        res.min_gap.append(min(st.gap[:a]))
-        res.min_gap_all.append(min(st.gap))
+        res.min_gap.append(min(gaps[:a]))
+        res.min_gap_all.append(min(gaps_all))
+        if mode == "verify" and cands:
+            # the cache past L holds the last forward's K/V: commit the
+            # accepted tokens' own
+            sess.forward(toks[:a], L, rows=[])
         L += a
         res.iterations += 1
         if stop or len(res.tokens) >= max_new:
@@ -435,6 +512,11 @@ def jacobi_decode(model: OracleModel, prompt: Sequence[int], n: int, max_new: in
             block = st.pred[a - 1:] + [g(it, i) for i in range(m - a + 1, m)]
             if mode == "lookahead":
                 block = ngram_pool_step(pool, st.pred, a, block, ngram)
+        elif mode == "verify":
+            # the committed run's next head, then the block's own predictions
+            # for the positions after it (refill when the block won)
+            block = [pred[a - 1]] + st.pred[a:m] + [g(it, i) for i in range(max(1, m - a + 1), m)]
+            ngram_pool_push(pool, st.pred, ngram, ncand)
         elif a == m:
             block = [st.pred[m - 1]] + [g(it, i) for i in range(1, n)]
         else:

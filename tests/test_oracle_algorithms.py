@@ -207,3 +207,123 @@ def test_lookahead_decode_equals_ar(tiny, n, ngram, seed):
         assert jr.tokens == ar.tokens
         assert all(a >= 1 for a in jr.accepted)
         assert sum(jr.accepted) == 40
+
+
+# ---- the same combination with a verification branch of several n-grams
+
+def test_ngram_pool_push_worked_example():
+    """Hand-worked pool updates with trigrams and at most two values a key:
+    a key keeps its distinct values most recent first, an n-gram entered again
+    moves to the front, and a third distinct value drops the oldest."""
+    pool = {}
+    orc.ngram_pool_push(pool, [5, 6, 7, 6, 7, 8], 3, 2)
+    assert pool == {5: [(6, 7)], 6: [(7, 8), (7, 6)], 7: [(6, 7)]}
+    orc.ngram_pool_push(pool, [6, 7, 6, 9], 3, 2)
+    assert pool[6] == [(7, 6), (7, 8)] and pool[7] == [(6, 9), (6, 7)]
+    orc.ngram_pool_push(pool, [6, 1, 1], 3, 2)
+    assert pool[6] == [(1, 1), (7, 6)]
+    # fewer predictions than the n-gram: nothing enters
+    orc.ngram_pool_push(pool, [2, 3], 3, 2)
+    assert 2 not in pool
+
+
+def test_verify_candidates_brute_force_micro_model(micro):
+    """Every two-token candidate after the head of a micro model, verified in
+    one call: each accepted count equals the count from Eq. 3's rows evaluated
+    by fresh full forwards, so no candidate sees another's K/V."""
+    m = micro
+    V = MICRO.vocab
+    prompt = [3, 1, 4, 1, 5]
+    ar = orc.ar_decode(m, prompt, 4)
+    head = ar.tokens[0]
+    cands = [[g1, g2] for g1 in range(V) for g2 in range(V)]
+    s = m.session(16)
+    s.forward(prompt, 0, rows=[])
+    res = orc.verify_candidates(s, head, cands, len(prompt))
+    seen = set()
+    for c, (a, q, gaps) in zip(cands, res):
+        assert a == _definitional_accept(m, prompt, [head] + c)
+        assert q[0] == ar.tokens[1] and len(q) == len(gaps) == 3
+        seen.add(a)
+    assert seen == {1, 2, 3}
+    # the AR continuation is accepted whole, and predicts the token after it
+    (a, q, _), = orc.verify_candidates(s, head, [ar.tokens[1:3]], len(prompt))
+    assert a == 3 and q == ar.tokens[1:4]
+
+
+@pytest.mark.parametrize("n,ngram,ncand,seed", [(8, 3, 4, 2), (8, 5, 2, 3), (16, 4, 4, 4), (4, 2, 1, 5)])
+def test_verify_decode_equals_ar(tiny, n, ngram, ncand, seed):
+    """A candidate's tokens are committed only as far as the model verifies
+    them, with their own K/V, so the decode is the greedy AR output
+    (Sec. 3.1); on this model's repeating continuations some iterations
+    commit a candidate, and then more tokens than the block would have."""
+    cfg, m = tiny
+    won = 0
+    for pl in (32, 17, 9):
+        prompt = syn.make_prompts(cfg.vocab, [pl], seed=seed)[0]
+        ar = orc.ar_decode(m, prompt, 48)
+        jr = orc.jacobi_decode(m, prompt, n, 48, seed=seed, mode="verify", ngram=ngram, ncand=ncand,
+                               record=True)
+        assert jr.tokens == ar.tokens
+        assert all(a >= 1 for a in jr.accepted) and sum(jr.accepted) == 48
+        assert len(jr.branch) == len(jr.candidates) == jr.iterations
+        for br, cands in zip(jr.branch, jr.candidates):
+            assert len(cands) <= ncand and all(len(c) == ngram - 1 for c in cands)
+            assert -1 <= br < len(cands)
+        won += sum(1 for br in jr.branch if br >= 0)
+    assert won >= 1
+
+
+def test_verify_without_pool_entries_is_refill(tiny):
+    """With n-grams longer than the block nothing enters the pool, no
+    candidate is verified, and the decode is the refill decode iteration for
+    iteration."""
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [17], seed=2)[0]
+    rf = orc.jacobi_decode(m, prompt, 8, 40, seed=3, mode="refill", record=True)
+    vr = orc.jacobi_decode(m, prompt, 8, 40, seed=3, mode="verify", ngram=9, ncand=4, record=True)
+    assert vr.trajectory == rf.trajectory and vr.accepted == rf.accepted
+    assert vr.branch == [-1] * vr.iterations and all(c == [] for c in vr.candidates)
+
+
+def test_verify_eos_inside_a_candidate(tiny):
+    """An EOS inside a committed candidate ends the decode at the EOS, as for
+    the block (Alg. 1's stop rule)."""
+    cfg, m = tiny
+    prompt = syn.make_prompts(cfg.vocab, [17], seed=2)[0]
+    jr = orc.jacobi_decode(m, prompt, 8, 48, seed=3, mode="verify", ngram=3, ncand=4)
+    ar_full = orc.ar_decode(m, prompt, 48).tokens
+    # the first token that a candidate committed beyond the head
+    pos, k = 0, None
+    for a, br in zip(jr.accepted, jr.branch):
+        if br >= 0 and a >= 2:
+            k = pos + 1
+            break
+        pos += a
+    assert k is not None
+    eos = ar_full[k]
+    first = ar_full.index(eos)
+    got = orc.jacobi_decode(m, prompt, 8, 48, seed=3, mode="verify", ngram=3, ncand=4, eos_id=eos)
+    assert got.tokens == ar_full[:first + 1]
+    assert got.tokens == orc.ar_decode(m, prompt, 48, eos_id=eos).tokens
+
+
+def test_verify_candidates_come_from_earlier_iterations(tiny):
+    """Sec. 3.3: candidates are n-grams generated in previous iterations.
+    Every n-gram verified at iteration i follows its head in the predictions
+    of some iteration before i, and the first iteration verifies none."""
+    cfg, m = tiny
+    ngram = 3
+    for pl, seed in ((17, 2), (9, 3)):
+        prompt = syn.make_prompts(cfg.vocab, [pl], seed=seed)[0]
+        jr = orc.jacobi_decode(m, prompt, 8, 48, seed=seed, mode="verify", ngram=ngram, ncand=4,
+                               record=True, keep_steps=True)
+        assert jr.candidates[0] == []
+        checked = 0
+        for i, (block, cands) in enumerate(zip(jr.trajectory, jr.candidates)):
+            earlier = {tuple(st.pred[k:k + ngram]) for st in jr.steps[:i]
+                       for k in range(len(st.pred) - ngram + 1)}
+            for c in cands:
+                assert (block[0], *c) in earlier, f"iteration {i}"
+                checked += 1
+        assert checked >= 1
